@@ -1,0 +1,496 @@
+"""Float64 CPU oracle for the ACRL vocabulary-wide hot path.
+
+TEST INFRASTRUCTURE ONLY.  This module exists so that the CUDA path can be
+checked against a plain, slow, obviously correct statement of what the paper
+defines.  Only the test-suite, the smoke check and the CPU-baseline leg of the
+benchmark may import it; the library and its Python binding never do.  It
+shares no code, header, constant table or helper with the CUDA path and
+imports nothing from it.
+
+Paper: "ACRL: Adaptive Control of Training-Inference Discrepancy for Stable
+Reinforcement Learning" (arXiv 2607.24062).  Every function below cites the
+passage it follows.  Everything is computed in float64 with numpy; bf16 logits
+are widened to float64 exactly (bf16 is a subset of float64).
+
+Where the paper is silent the oracle takes these readings (they are also the
+readings of the CUDA path; each is listed with its reason in the design notes):
+  * d is an absolute difference of probabilities, not of log-probabilities
+    (Eq. distance_metric, Sec. 4.1).
+  * Y defaults to the group form (1/G) sum_i (1/|a_i|) sum_t d, literally the
+    formula after Eq. ACRL; per-sequence and whole-batch forms are options.
+  * Sequences with no valid token are left out of Y_g and of G_g; a group with
+    no valid sequence is left out of the prompt count.
+  * GRPO std uses ddof=1 plus adv_eps; a group of one response gets mean 0 and
+    std 1 (so A = R) unless the ZERO rule is chosen.
+  * sign(0) = 0, so A = 0 gives alpha = 0 and rho = 1.
+  * min(rho, C) is evaluated as exp(min(alpha*lr, ln C)); the MIS indicator
+    1{rho_i <= C} as S_i <= ln C.
+  * X is the mean of Y_g over the prompts of the first `calib_steps` batches
+    (Sec. 4.1, "compiled before training"; Sec. 5.1 takes it from step 0), then
+    frozen.  If X <= 0 the controller sets alpha = 0 and raises a flag.
+  * The clip tie r = 1 +/- eps keeps the unclipped branch.
+  * Masked tokens contribute nothing: their outputs are 0 and their gradient
+    row is 0.  A row whose coefficient is 0 has a zero gradient row.
+  * Any non-finite logit in a valid row makes that row's lse/logp/entropy NaN
+    and sets a flag; a sampled id outside [0, V) gives logp = 0, a zero
+    gradient row and a flag.
+
+Parity status: every function here is pinned by tests that do not re-use its
+own formulas (brute force, closed forms, invariants, finite differences and
+the sign table of Sec. 4.2).  The paper prints no worked numeric example, so no
+function is pinned to a number the paper prints.
+"""
+
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+
+# Weight modes (Sec. 2.2 TIS / MIS, Sec. 4.1 ACRL, plain GRPO).
+MODE_NONE, MODE_TIS, MODE_MIS, MODE_ACRL = 0, 1, 2, 3
+# Granularity of the current discrepancy Y.
+Y_GROUP, Y_SEQUENCE, Y_BATCH = 0, 1, 2
+# Loss aggregation.
+AGG_SEQ_MEAN_TOKEN_MEAN, AGG_TOKEN_MEAN = 0, 1
+# GRPO rule for a group with a single response.
+SINGLETON_MEAN0_STD1, SINGLETON_ZERO = 0, 1
+
+# Data-dependent error bits (the oracle's own copy of the library's meaning).
+FLAG_BAD_ID = 1
+FLAG_NONFINITE = 2
+FLAG_BAD_OFFSETS = 4
+FLAG_X_NONPOS = 8
+
+
+@dataclass
+class Params:
+    """Hyper-parameters.  Defaults: gamma=0.65 and C=3 (Sec. 5.1); eps is not
+    given by the paper, 0.2 is the usual GRPO value."""
+
+    gamma: float = 0.65
+    C: float = 3.0
+    clip_eps: float = 0.2
+    adv_eps: float = 1e-6
+    mode: int = MODE_ACRL
+    y_gran: int = Y_GROUP
+    agg: int = AGG_SEQ_MEAN_TOKEN_MEAN
+    adv_ddof: int = 1
+    singleton_rule: int = SINGLETON_MEAN0_STD1
+    calib_steps: int = 1
+    X_init: float = 0.0
+
+
+@dataclass
+class ControllerState:
+    """The controller's whole state: the reference X and its calibration sums
+    (Sec. 4.1: X is built before training and then kept fixed)."""
+
+    X: float = 0.0
+    calib_sum: float = 0.0
+    calib_count: int = 0
+    calib_done_steps: int = 0
+    step: int = 0
+    calibrated: bool = False
+    flags: int = 0
+
+
+def controller_init(params: Params) -> ControllerState:
+    """A given X (> 0) skips calibration, as with the printed X values of
+    Sec. 5.1; otherwise X is measured on the first batches."""
+    st = ControllerState()
+    if params.X_init > 0:
+        st.X = float(params.X_init)
+        st.calibrated = True
+    return st
+
+
+# --------------------------------------------------------------------------
+# bf16 handling
+# --------------------------------------------------------------------------
+
+def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Widen raw bf16 bit patterns (uint16) to float64 exactly: a bf16 value is
+    the upper half of the float32 with the same bits."""
+    u = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return u.view(np.float32).astype(np.float64)
+
+
+# --------------------------------------------------------------------------
+# a1: log-softmax, sampled-token log-prob, entropy
+# --------------------------------------------------------------------------
+
+def token_stats(z: np.ndarray, ids: np.ndarray, mask: np.ndarray | None):
+    """Per row t: lse_t = log sum_j exp(z_tj); logp_t = z_{t,a_t} - lse_t is
+    log pi(a_t | q, a_<t) as used in r (Eq. grpo_objective), rho (Eq. TIS) and
+    d (Eq. distance_metric); H_t = -sum_j p_tj log p_tj is the token entropy
+    the paper tracks during training (Sec. 5.1 figures).
+
+    z: float64 [T, V].  Returns (lse, logp, H, flags)."""
+    z = np.asarray(z, dtype=np.float64)
+    T, V = z.shape
+    ids = np.asarray(ids).astype(np.int64)
+    m = np.ones(T, dtype=bool) if mask is None else (np.asarray(mask) != 0)
+    lse = np.zeros(T)
+    logp = np.zeros(T)
+    H = np.zeros(T)
+    flags = 0
+    for t in range(T):
+        if not m[t]:
+            continue
+        row = z[t]
+        if not np.all(np.isfinite(row)):
+            lse[t] = logp[t] = H[t] = np.nan
+            flags |= FLAG_NONFINITE
+            continue
+        zmax = row.max()
+        lse[t] = zmax + np.log(np.sum(np.exp(row - zmax)))
+        logq = row - lse[t]                 # log-softmax of the row
+        p = np.exp(logq)
+        H[t] = -np.sum(p * logq)
+        a = ids[t]
+        if 0 <= a < V:
+            logp[t] = logq[a]
+        else:
+            logp[t] = 0.0
+            flags |= FLAG_BAD_ID
+    return lse, logp, H, flags
+
+
+def token_stats_bruteforce(z, ids, mask=None):
+    """The same quantities with plain Python loops and math.fsum; only for
+    small V (a pin for `token_stats`)."""
+    T = len(z)
+    out_lse, out_logp, out_H = [], [], []
+    for t in range(T):
+        if mask is not None and not mask[t]:
+            out_lse.append(0.0)
+            out_logp.append(0.0)
+            out_H.append(0.0)
+            continue
+        row = [float(v) for v in z[t]]
+        big = max(row)
+        s = math.fsum(math.exp(v - big) for v in row)
+        lse = big + math.log(s)
+        probs = [math.exp(v - lse) for v in row]
+        ent = -math.fsum(p * math.log(p) for p in probs if p > 0.0)
+        out_lse.append(lse)
+        out_logp.append(math.log(probs[int(ids[t])]))
+        out_H.append(ent)
+    return np.array(out_lse), np.array(out_logp), np.array(out_H)
+
+
+# --------------------------------------------------------------------------
+# a2/a3: log-ratio, distance, masked segmented aggregates
+# --------------------------------------------------------------------------
+
+def _check_offsets(seq_offsets, group_offsets, T):
+    so = np.asarray(seq_offsets, dtype=np.int64)
+    go = np.asarray(group_offsets, dtype=np.int64)
+    S = len(so) - 1
+    ok = (len(so) >= 1 and so[0] == 0 and so[-1] == T and np.all(np.diff(so) >= 0)
+          and len(go) >= 1 and go[0] == 0 and go[-1] == S and np.all(np.diff(go) >= 0))
+    return so, go, bool(ok)
+
+
+def seq_discrepancy(logp_pi, logp_mu, mask, seq_offsets, group_offsets, entropy=None):
+    """Per token: lr_t = log pi_old(a_t) - log mu(a_t) (the log of rho in
+    Eq. TIS) and d_t = |pi_old(a_t) - mu(a_t)| (Eq. distance_metric).
+    Per sequence i: n_i = |a_i| (valid tokens), D_i = (1/n_i) sum_t d_t, the
+    MIS log-ratio S_i = sum_t lr_t = log rho_i (Eq. MIS), max/sum/sum-of-squares
+    of d and the mean entropy.  Per group g: G_g valid sequences and
+    Y_g = (1/G_g) sum_i D_i (the current discrepancy Y defined after Eq. ACRL).
+    Batch: token mean/max/std of d (the curves of Sec. 5.1), the prompt mean of
+    Y_g (the step discrepancy of the X-evolution table), token-mean entropy and
+    log-ratio.
+
+    Returns (lr, d, seq, grp, batch, flags) with seq/grp/batch dicts."""
+    pi = np.asarray(logp_pi, dtype=np.float64)
+    mu = np.asarray(logp_mu, dtype=np.float64)
+    T = len(pi)
+    m = np.ones(T, dtype=bool) if mask is None else (np.asarray(mask) != 0)
+    so, go, ok = _check_offsets(seq_offsets, group_offsets, T)
+    flags = 0 if ok else FLAG_BAD_OFFSETS
+    S, Gn = len(so) - 1, len(go) - 1
+
+    lr = np.where(m, pi - mu, 0.0)
+    d = np.where(m, np.abs(np.exp(pi) - np.exp(mu)), 0.0)
+    Hm = None if entropy is None else np.where(m, np.asarray(entropy, dtype=np.float64), 0.0)
+
+    seq = {k: np.zeros(S) for k in ("mean_d", "max_d", "sum_d", "sum_d2", "sum_lr", "mean_H")}
+    seq["n"] = np.zeros(S, dtype=np.int64)
+    seq["group"] = np.full(S, -1, dtype=np.int64)
+    for g in range(Gn):
+        seq["group"][go[g]:go[g + 1]] = g
+    for i in range(S):
+        sl = slice(so[i], so[i + 1])
+        mi = m[sl]
+        n = int(mi.sum())
+        seq["n"][i] = n
+        if n == 0:
+            continue
+        di = d[sl][mi]
+        seq["sum_d"][i] = di.sum()
+        seq["sum_d2"][i] = (di * di).sum()
+        seq["max_d"][i] = di.max()
+        seq["mean_d"][i] = di.sum() / n
+        seq["sum_lr"][i] = lr[sl][mi].sum()
+        if Hm is not None:
+            seq["mean_H"][i] = Hm[sl][mi].sum() / n
+
+    grp = {"n_valid_seqs": np.zeros(Gn, dtype=np.int64), "n_tokens": np.zeros(Gn, dtype=np.int64),
+           "Y": np.zeros(Gn)}
+    for g in range(Gn):
+        members = range(go[g], go[g + 1])
+        valid = [i for i in members if seq["n"][i] > 0]
+        grp["n_valid_seqs"][g] = len(valid)
+        grp["n_tokens"][g] = sum(int(seq["n"][i]) for i in members)
+        if valid:
+            grp["Y"][g] = sum(seq["mean_d"][i] for i in valid) / len(valid)
+
+    valid_g = grp["n_valid_seqs"] > 0
+    N = int(m.sum())
+    dv = d[m]
+    batch = {
+        "n_tokens": N,
+        "n_groups_valid": int(valid_g.sum()),
+        "n_seqs_valid": int((seq["n"] > 0).sum()),
+        "d_mean": float(dv.mean()) if N else 0.0,
+        "d_max": float(dv.max()) if N else 0.0,
+        "d_std": float(dv.std()) if N else 0.0,
+        "Y_sum": float(grp["Y"][valid_g].sum()),
+        "Y_mean": float(grp["Y"][valid_g].mean()) if valid_g.any() else 0.0,
+        "H_mean": float(Hm[m].mean()) if (Hm is not None and N) else 0.0,
+        "lr_mean": float(lr[m].mean()) if N else 0.0,
+    }
+    return lr, d, seq, grp, batch, flags
+
+
+# --------------------------------------------------------------------------
+# a4: GRPO advantage
+# --------------------------------------------------------------------------
+
+def grpo_advantage(rewards, group_offsets, params: Params):
+    """A_i = (R_i - mean_g R) / std_g R over the responses of one prompt
+    (Sec. 2, the definition under Eq. grpo_objective), with std taken with
+    `adv_ddof` degrees of freedom and `adv_eps` added to it."""
+    R = np.asarray(rewards, dtype=np.float64)
+    go = np.asarray(group_offsets, dtype=np.int64)
+    A = np.zeros(len(R))
+    for g in range(len(go) - 1):
+        r = R[go[g]:go[g + 1]]
+        G = len(r)
+        if G == 0:
+            continue
+        if G == 1:
+            A[go[g]] = r[0] if params.singleton_rule == SINGLETON_MEAN0_STD1 else 0.0
+            continue
+        mean = r.sum() / G
+        var = ((r - mean) ** 2).sum() / (G - params.adv_ddof) if G > params.adv_ddof else 0.0
+        A[go[g]:go[g + 1]] = (r - mean) / (math.sqrt(var) + params.adv_eps)
+    return A
+
+
+# --------------------------------------------------------------------------
+# a5: controller step and importance weights
+# --------------------------------------------------------------------------
+
+def controller_step(state: ControllerState, params: Params, lr, mask, seq_offsets, group_offsets,
+                    seq, grp, batch, adv):
+    """Calibrate or apply the reference X (Sec. 4.1), then the per-sequence
+    exponent alpha_i = gamma * sign(A_i) * (1 - Y/X) (Sec. 4.1, after
+    Eq. ACRL) and per-token weights:
+      ACRL: min(rho_t, C) with rho_t = (pi_old/mu)^alpha_i   (Eq. ACRL)
+      TIS : min(pi_old/mu, C)                                (Eq. TIS)
+      MIS : rho_i * 1{rho_i <= C}, rho_i = prod_t pi_old/mu   (Eq. MIS)
+      NONE: 1                                                (Eq. grpo_objective)
+    Returns (weight [T], alpha [S], new_state, info dict, flags).  `state` is
+    not modified."""
+    st = ControllerState(**vars(state))
+    lr = np.asarray(lr, dtype=np.float64)
+    T = len(lr)
+    m = np.ones(T, dtype=bool) if mask is None else (np.asarray(mask) != 0)
+    so = np.asarray(seq_offsets, dtype=np.int64)
+    S = len(so) - 1
+    A = np.asarray(adv, dtype=np.float64)
+    flags = 0
+
+    applying = True
+    if not st.calibrated:
+        st.calib_sum += batch["Y_sum"]
+        st.calib_count += batch["n_groups_valid"]
+        st.calib_done_steps += 1
+        if st.calib_done_steps >= params.calib_steps:
+            st.X = st.calib_sum / st.calib_count if st.calib_count > 0 else 0.0
+            st.calibrated = True
+        else:
+            applying = False
+    st.step += 1
+
+    X = st.X
+    if params.mode == MODE_ACRL and applying and not X > 0:
+        flags |= FLAG_X_NONPOS
+
+    logC = math.log(params.C)
+    alpha = np.zeros(S)
+    w = np.zeros(T)
+    n_trunc = 0
+    for i in range(S):
+        n_i = int(seq["n"][i])
+        if params.mode == MODE_TIS or params.mode == MODE_MIS:
+            alpha[i] = 1.0
+        elif params.mode == MODE_ACRL and applying and X > 0 and n_i > 0:
+            if params.y_gran == Y_GROUP:
+                Y = grp["Y"][seq["group"][i]]
+            elif params.y_gran == Y_SEQUENCE:
+                Y = seq["mean_d"][i]
+            else:
+                Y = batch["Y_mean"]
+            alpha[i] = params.gamma * np.sign(A[i]) * (1.0 - Y / X)
+        for t in range(so[i], so[i + 1]):
+            if not m[t]:
+                continue
+            if params.mode == MODE_NONE:
+                w[t] = 1.0
+            elif params.mode == MODE_MIS:
+                S_i = seq["sum_lr"][i]
+                w[t] = math.exp(S_i) if S_i <= logC else 0.0
+                n_trunc += S_i > logC
+            else:
+                log_rho = alpha[i] * lr[t]
+                w[t] = math.exp(min(log_rho, logC))
+                n_trunc += log_rho > logC
+    N = int(m.sum())
+    valid_seq = np.asarray(seq["n"]) > 0
+    info = {
+        "X": X,
+        "trunc_frac": n_trunc / N if N else 0.0,
+        "w_mean": float(w[m].mean()) if N else 0.0,
+        "alpha_mean": float(alpha[valid_seq].mean()) if valid_seq.any() else 0.0,
+    }
+    st.flags |= flags
+    return w, alpha, st, info, flags
+
+
+# --------------------------------------------------------------------------
+# a6: policy loss and its gradient with respect to the logits
+# --------------------------------------------------------------------------
+
+def _seq_of_rows(so, T):
+    owner = np.full(T, -1, dtype=np.int64)
+    for i in range(len(so) - 1):
+        owner[so[i]:so[i + 1]] = i
+    return owner
+
+
+def loss_grad_logits(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch,
+                     params: Params, rows=None):
+    """Loss of Eq. ACRL (Eq. TIS / Eq. MIS / Eq. grpo_objective for the other
+    modes: the weight is the only difference) and its gradient w.r.t. the
+    logits.  Per valid token, with r_t = exp(logp_t - old_logp_t) (r = 1 when
+    `old_logp` is None, the one-update-per-rollout setting of App. A):
+        loss_t = -w_t * min(r_t A_i, clip(r_t, 1-eps, 1+eps) A_i) / norm_t
+    with norm_t = Q_eff * G_g * n_i (the 1/G sum_i 1/|a_i| sum_t of the
+    objective, averaged over prompts) or the valid-token count (TOKEN_MEAN).
+    The weight w_t is a constant (it is built from theta_old).  By the chain
+    rule, d logp_t / d z_tj = 1[j = a_t] - p_tj and dr/dz = r dlogp/dz, so
+        dL/dz_tj = coef_t (p_tj - 1[j = a_t]),
+        coef_t = w_t g_t r_t A_i / norm_t,
+    where g_t = 1 when the unclipped branch is the minimum (A >= 0 and
+    r <= 1+eps, or A < 0 and r >= 1-eps) and 0 otherwise.
+
+    z: float64 [T, V] (or only the rows listed in `rows`, in that order).
+    lse: None to recompute from z.  Returns (grad [len(rows), V],
+    token_loss [T] (NaN where not computed), loss over the computed rows)."""
+    z = np.asarray(z, dtype=np.float64)
+    so = np.asarray(seq_offsets, dtype=np.int64)
+    T = len(np.asarray(weight))
+    rows = np.arange(T) if rows is None else np.asarray(rows, dtype=np.int64)
+    V = z.shape[1]
+    m = np.ones(T, dtype=bool) if mask is None else (np.asarray(mask) != 0)
+    ids = np.asarray(ids).astype(np.int64)
+    A = np.asarray(adv, dtype=np.float64)
+    w = np.asarray(weight, dtype=np.float64)
+    owner = _seq_of_rows(so, T)
+    eps = params.clip_eps
+    grad = np.zeros((len(rows), V))
+    token_loss = np.full(T, np.nan)
+    total = []
+    for k, t in enumerate(rows):
+        i = owner[t]
+        a = ids[t]
+        if i < 0 or not m[t] or not (0 <= a < V):
+            token_loss[t] = 0.0
+            total.append(0.0)
+            continue
+        row = z[k]
+        if lse is None:
+            top = row.max()
+            lse_t = top + np.log(np.sum(np.exp(row - top)))
+        else:
+            lse_t = float(lse[t])
+        logp_t = row[a] - lse_t
+        r = 1.0 if old_logp is None else math.exp(logp_t - float(old_logp[t]))
+        g_idx = int(seq["group"][i])
+        if params.agg == AGG_TOKEN_MEAN:
+            norm = float(batch["n_tokens"])
+        else:
+            norm = float(batch["n_groups_valid"]) * float(grp["n_valid_seqs"][g_idx]) * float(seq["n"][i])
+        Ai = A[i]
+        rc = min(max(r, 1.0 - eps), 1.0 + eps)
+        surrogate = min(r * Ai, rc * Ai)
+        token_loss[t] = -w[t] * surrogate / norm
+        total.append(token_loss[t])
+        gate = (Ai >= 0 and r <= 1.0 + eps) or (Ai < 0 and r >= 1.0 - eps)
+        coef = w[t] * (1.0 if gate else 0.0) * r * Ai / norm
+        if coef == 0.0:
+            continue
+        p = np.exp(row - lse_t)
+        p[a] -= 1.0
+        grad[k] = coef * p
+    return grad, token_loss, math.fsum(total)
+
+
+# --------------------------------------------------------------------------
+# whole step (for tests and the CPU baseline)
+# --------------------------------------------------------------------------
+
+@dataclass
+class StepResult:
+    lse: np.ndarray
+    logp: np.ndarray
+    H: np.ndarray
+    lr: np.ndarray
+    d: np.ndarray
+    seq: dict
+    grp: dict
+    batch: dict
+    adv: np.ndarray
+    weight: np.ndarray
+    alpha: np.ndarray
+    state: ControllerState
+    info: dict
+    grad: np.ndarray
+    token_loss: np.ndarray
+    loss: float
+    flags: int = 0
+    extra: dict = field(default_factory=dict)
+
+
+def step(z, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, params: Params,
+         state: ControllerState | None = None):
+    """One on-policy pass in the paper's order: log-probs and entropy of pi,
+    discrepancy statistics against mu, GRPO advantages, the controller, then
+    the loss gradient with respect to the logits (theta = theta_old, r = 1)."""
+    if state is None:
+        state = controller_init(params)
+    lse, logp, H, f1 = token_stats(z, ids, mask)
+    lr, d, seq, grp, batch, f2 = seq_discrepancy(logp, logp_mu, mask, seq_offsets, group_offsets, H)
+    adv = grpo_advantage(rewards, group_offsets, params)
+    w, alpha, st, info, f3 = controller_step(state, params, lr, mask, seq_offsets, group_offsets,
+                                             seq, grp, batch, adv)
+    grad, tl, loss = loss_grad_logits(z, ids, mask, lse, None, adv, w, seq_offsets, seq, grp, batch,
+                                      params)
+    return StepResult(lse, logp, H, lr, d, seq, grp, batch, adv, w, alpha, st, info, grad, tl, loss,
+                      f1 | f2 | f3)
