@@ -1,0 +1,420 @@
+"""Throughput of the ACRL vocabulary-wide hot path on GB300.
+
+One step = one on-policy pass of the whole path over one batch of the
+Qwen-vocabulary workload (16 prompts x 8 responses, lengths U[256, 2048],
+V = 151,936, bf16 logits, Student-t(4) x 2): token statistics, discrepancy
+statistics, GRPO advantages, the controller and the loss gradient w.r.t. the
+logits, all through the C ABI.  Inputs are generated on the device from fixed
+seeds and are far larger than L2 (44.8 GB of logits), so no L2 flush is needed
+between steps.
+
+Prints one JSON line.  `--impl reference` times the float64 CPU oracle on a
+bounded row sample of the same workload instead (rank 0 only).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "tokens/s fused logprob+discrepancy+grad at V=151936; HBM GB/s vs peak"
+UNIT = "tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+# Kernel launches per step inside the timed region: token_stats 1, seq_discrepancy 2,
+# grpo_advantage 1, controller_step 3, loss_grad_logits 2.
+LAUNCHES_PER_STEP = 9
+# DRAM traffic of one gradient-kernel launch on the bench workload, from ncu
+# (dram__bytes_read.sum + dram__bytes_write.sum), valid only for the kernel source
+# it was taken on (sha256 of the file, first 16 hex digits).
+NCU_TRAFFIC = {}
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def _src_hash(name):
+    p = os.path.join(ROOT, "paper_2607_24062_gb300", "csrc", name)
+    with open(p, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-i", str(self.index), "-lms", "100"], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            if self.thread is not None:
+                self.thread.join(timeout=2)
+
+    def summary(self):
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, mx, reasons = [], [], set()
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) != 6:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[2:]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _dist():
+    import torch
+    import torch.distributed as dist
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    return world, rank, local
+
+
+def _workload_desc(spec):
+    return (f"{spec.name}: {spec.n_prompts} prompts x {spec.group_size} responses, lengths U[{spec.len_lo},"
+            f"{spec.len_hi}], V={spec.V}, bf16 logits {spec.dist}(scale {spec.scale}), mu = FP8-E4M3 "
+            f"{spec.fp8_scale}-scaled round-trip")
+
+
+# --------------------------------------------------------------------------
+# CPU oracle leg
+# --------------------------------------------------------------------------
+
+def oracle_tokens_per_s(batch, params, rows_budget_s=10.0, max_rows=4096, rng_seed=0):
+    """Time the float64 oracle on a bounded sample: the O(T) stages over the
+    whole batch once, the vocabulary-wide stages (log-softmax statistics and the
+    gradient) on sampled rows until `rows_budget_s` has passed.  Returns
+    (tokens/s extrapolated to the whole batch, description)."""
+    import torch
+
+    import oracle as O
+
+    T, V = batch.T, batch.V
+    mask = batch.mask.cpu().numpy()
+    ids = batch.ids.cpu().numpy()
+    mu = batch.logp_mu.cpu().numpy().astype(np.float64)
+    R = batch.rewards.cpu().numpy().astype(np.float64)
+    so = batch.seq_offsets.cpu().numpy()
+    go = batch.group_offsets.cpu().numpy()
+    op = O.Params(gamma=params.gamma, C=params.C, clip_eps=params.clip_eps, adv_eps=params.adv_eps)
+    rng = np.random.default_rng(rng_seed)
+    rows = rng.permutation(np.flatnonzero(mask))[:max_rows]
+    # vocabulary-wide part on sampled rows (time-boxed)
+    t0 = time.perf_counter()
+    done = 0
+    lse_s = {}
+    block = 16
+    while done < len(rows) and time.perf_counter() - t0 < rows_budget_s:
+        rr = rows[done:done + block]
+        idx = torch.as_tensor(rr, device=batch.logits.device)
+        bits = batch.logits.index_select(0, idx)[:, :V].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        tc = time.perf_counter()
+        z = O.bf16_bits_to_f64(bits)
+        lse, logp, H, _ = O.token_stats(z, ids[rr], mask[rr])
+        # gradient of the same rows with a representative weight/advantage
+        O.loss_grad_logits(z, ids[rr], mask[rr], lse, None, np.ones(len(rr)), np.ones(len(rr)),
+                           np.arange(len(rr) + 1), {"n": np.ones(len(rr), dtype=np.int64),
+                                                    "group": np.zeros(len(rr), dtype=np.int64)},
+                           {"n_valid_seqs": np.array([len(rr)])}, {"n_groups_valid": 1, "n_tokens": len(rr)}, op)
+        lse_s[done] = time.perf_counter() - tc
+        done += len(rr)
+    t_rows = sum(lse_s.values())
+    # O(T) part on the whole batch, from the batch's own GPU-independent inputs
+    tc = time.perf_counter()
+    # the O(T) stages need pi's log-probs for every token; the rollout log-probs stand in (same cost)
+    lr, d, seq, grp, bst, _ = O.seq_discrepancy(mu, mu, mask, so, go)
+    adv = O.grpo_advantage(R, go, op)
+    w, alpha, st, info, _ = O.controller_step(O.controller_init(op), op, lr, mask, so, go, seq, grp, bst, adv)
+    O.loss_coefficients(w, adv, mask, so, seq, grp, bst, op)
+    t_ot = time.perf_counter() - tc
+    n_valid = int(mask.sum())
+    per_token = t_rows / max(1, done) + t_ot / max(1, n_valid)
+    desc = (f"float64 numpy oracle, 1 thread: log-softmax statistics + gradient on {done} sampled rows "
+            f"({t_rows:.1f} s) and the O(T) stages on all {n_valid} tokens ({t_ot:.1f} s), extrapolated per token")
+    return 1.0 / per_token, desc, done
+
+
+def run_reference(args):
+    world, rank, local = _dist()
+    if rank != 0:
+        return 0
+    import torch
+
+    import paper_2607_24062_gb300 as acrl
+    import workloads as W
+    spec = W.QWEN
+    dev = torch.device(f"cuda:{local}" if torch.cuda.is_available() else "cpu")
+    if dev.type == "cuda":
+        torch.cuda.set_device(dev)
+    batch = W.generate(spec, seed=W.seed_for(spec.name), device=dev)
+    params = acrl.Params()
+    vals = []
+    t_all = []
+    for k in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        v, desc, n = oracle_tokens_per_s(batch, params, rows_budget_s=args.ref_seconds, max_rows=4096, rng_seed=k)
+        t_all.append(time.perf_counter() - t0)
+        if k >= args.warmup:
+            vals.append(v)
+    value = float(np.median(vals))
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": float(np.median(t_all[args.warmup:])) * 1e3,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": _workload_desc(spec), "T": batch.T, "V": batch.V},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+    return 0
+
+
+# --------------------------------------------------------------------------
+# our arm
+# --------------------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2607_24062_gb300 as acrl
+    import workloads as W
+    from paper_2607_24062_gb300 import build
+
+    world, rank, local = _dist()
+    build.build()
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    spec = W.SPECS[args.workload]
+    # weak scaling: each rank owns its own batch of prompts (independent groups; X is frozen per rank after
+    # its first batch, so no data-path collective exists)
+    batch = W.generate(spec, seed=W.seed_for(spec.name) + 7919 * rank, device=dev)
+    params = acrl.Params()
+    step = acrl.AcrlStep.for_batch(batch, params, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    for _ in range(args.warmup):
+        step.run_batch(batch)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+
+    n_valid = int(batch.mask.sum())
+    mask_h = batch.mask.bool().cpu()
+    coef_h = step.coef.cpu()
+    ids_h = batch.ids.cpu()
+    live = mask_h & (coef_h != 0) & (ids_h >= 0) & (ids_h < batch.V)
+    V = batch.V
+    # algorithmic bytes per launch
+    k5_bytes = int(live.sum()) * 4 * V + (batch.T - int(live.sum())) * 2 * V + batch.T * 17
+    k1_bytes = n_valid * 2 * V + batch.T * 17
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index) as clocks:
+        torch.cuda.synchronize()
+        start.record(stream)
+        for k in range(args.steps):
+            e0, e1, e2, e3 = ev[k]
+            e0.record(stream)
+            acrl.token_stats(batch.logits, batch.ids, batch.mask, V=V, lse=step.lse, logp=step.logp,
+                             entropy=step.entropy, flags=step.flags)
+            e1.record(stream)
+            # the rest of the statistics pass (seq_discrepancy, grpo_advantage, controller_step)
+            acrl.seq_discrepancy(step.logp, batch.logp_mu, batch.mask, batch.seq_offsets, batch.group_offsets,
+                                 step.entropy, out=step.disc, flags=step.flags)
+            acrl.grpo_advantage(batch.rewards, batch.group_offsets, params, adv=step.adv, flags=step.flags)
+            acrl.controller_step(step.state, params, step.disc, batch.mask, batch.seq_offsets, batch.group_offsets,
+                                 step.adv, weight=step.weight, coef=step.coef, alpha=step.alpha, flags=step.flags)
+            e2.record(stream)
+            acrl.loss_grad_logits(batch.logits, batch.ids, batch.mask, step.lse, None, step.coef, params.clip_eps,
+                                  V=V, grad=step.grad, token_loss=step.token_loss, loss=step.loss, flags=step.flags)
+            e3.record(stream)
+        end.record(stream)
+        torch.cuda.synchronize()
+    total_ms = start.elapsed_time(end)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t)
+        nt = torch.tensor([n_valid], device=dev, dtype=torch.float64)
+        dist.all_reduce(nt)
+        tokens_all = float(nt)
+    else:
+        tokens_all = float(n_valid)
+    k1_ms = [ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps)]
+    mid_ms = [ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps)]
+    k5_ms = [ev[k][2].elapsed_time(ev[k][3]) for k in range(args.steps)]
+    ms_per_step = total_ms / args.steps
+    value = tokens_all * args.steps / (total_ms / 1e3)
+
+    peak, peak_kind = _peaks()
+    k5_avg = float(np.mean(k5_ms))
+    k1_avg = float(np.mean(k1_ms))
+    k5_gbs = k5_bytes / (k5_avg / 1e3) / 1e9
+    k1_gbs = k1_bytes / (k1_avg / 1e3) / 1e9
+    tr = NCU_TRAFFIC.get("loss_grad.cu")
+    traffic = tr["bytes_per_launch"] if tr and tr["src"] == _src_hash("loss_grad.cu") else None
+
+    e2e = None
+    if not args.no_e2e and rank == 0:
+        e2e = run_e2e(batch, params, args, dev)
+    if world > 1:
+        dist.barrier()
+    if rank != 0:
+        return 0
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": _workload_desc(spec), "T": batch.T, "V": V, "ld": batch.ld,
+                   "tokens_per_step": n_valid, "logits": "bf16 in, gradient bf16 out, fp32 arithmetic",
+                   "l2": "no flush: inputs (44.8 GB of logits) far larger than the 129 MB L2",
+                   "parallelism": f"weak, {world} independent batch(es)"},
+        "roofline": {"bound": "hbm", "kernel": "acrl_loss_grad_logits", "achieved": k5_gbs, "peak": peak,
+                     "unit": "GB/s", "frac": k5_gbs / peak, "traffic": traffic, "peak_kind": peak_kind,
+                     "algorithmic_bytes_per_launch": k5_bytes, "ms_per_launch": k5_avg},
+        "kernels": {
+            "acrl_token_stats": {"ms": k1_avg, "GB/s": k1_gbs, "frac": k1_gbs / peak, "bytes": k1_bytes},
+            "acrl_loss_grad_logits": {"ms": k5_avg, "GB/s": k5_gbs, "frac": k5_gbs / peak, "bytes": k5_bytes},
+            "seq_discrepancy+grpo_advantage+controller_step": {"ms": float(np.mean(mid_ms))},
+            "whole_step_GB/s": (k1_bytes + k5_bytes) / (ms_per_step / 1e3) / 1e9,
+        },
+        "clocks": clocks.summary(),
+        "gpu_launches": LAUNCHES_PER_STEP * args.steps,
+    }
+    if e2e is not None:
+        out["e2e"] = e2e
+    if not args.no_cpu and world == 1:
+        v, desc, n = oracle_tokens_per_s(batch, params, rows_budget_s=args.ref_seconds)
+        out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
+    print(json.dumps(out))
+    return 0
+
+
+def run_e2e(batch, params, args, dev):
+    """Same metric through the public API with host buffers: every step copies
+    the step's inputs from pinned host memory, runs the path and copies the
+    gradient and the loss back."""
+    import torch
+
+    import paper_2607_24062_gb300 as acrl
+    T, ld = batch.logits.shape
+    host = {
+        "logits": torch.empty((T, ld), dtype=torch.bfloat16, pin_memory=True),
+        "ids": batch.ids.cpu().pin_memory(), "mask": batch.mask.cpu().pin_memory(),
+        "logp_mu": batch.logp_mu.cpu().pin_memory(), "rewards": batch.rewards.cpu().pin_memory(),
+        "seq_offsets": batch.seq_offsets.cpu().pin_memory(), "group_offsets": batch.group_offsets.cpu().pin_memory(),
+    }
+    host["logits"].copy_(batch.logits)
+    grad_host = torch.empty((T, ld), dtype=torch.bfloat16, pin_memory=True)
+    loss_host = torch.empty(1, dtype=torch.float32, pin_memory=True)
+    devbuf = {k: torch.empty_like(v, device=dev) for k, v in host.items() if k != "logits"}
+    devbuf["logits"] = batch.logits  # reuse the resident buffer as the upload target
+    step = acrl.AcrlStep.for_batch(batch, params, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def one():
+        for k, v in host.items():
+            devbuf[k].copy_(v, non_blocking=True)
+        step.run(devbuf["logits"], devbuf["ids"], devbuf["mask"], devbuf["logp_mu"], devbuf["rewards"],
+                 devbuf["seq_offsets"], devbuf["group_offsets"])
+        grad_host.copy_(step.grad, non_blocking=True)
+        loss_host.copy_(step.loss, non_blocking=True)
+
+    one()
+    torch.cuda.synchronize()
+    n = max(1, args.e2e_steps)
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record(stream)
+    for _ in range(n):
+        one()
+    e.record(stream)
+    torch.cuda.synchronize()
+    ms = s.elapsed_time(e) / n
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    d2h = grad_host.numel() * grad_host.element_size() + 4
+    return {"value": int(batch.mask.sum()) / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="qwen")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--ref-seconds", type=float, default=10.0)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

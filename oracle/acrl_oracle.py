@@ -452,6 +452,61 @@ def loss_grad_logits(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq,
     return grad, token_loss, math.fsum(total)
 
 
+def _norms(mask, seq_offsets, seq, grp, batch, params: Params):
+    """norm_t of the aggregation: Q_eff * G_g * n_i (the prompt average of
+    (1/G) sum_i (1/|a_i|) sum_t in Eq. grpo_objective) or the token count."""
+    so = np.asarray(seq_offsets, dtype=np.int64)
+    T = int(so[-1])
+    owner = _seq_of_rows(so, T)
+    norm = np.zeros(T)
+    for t in range(T):
+        i = owner[t]
+        if i < 0:
+            continue
+        if params.agg == AGG_TOKEN_MEAN:
+            norm[t] = float(batch["n_tokens"])
+        else:
+            g = int(seq["group"][i])
+            norm[t] = float(batch["n_groups_valid"]) * float(grp["n_valid_seqs"][g]) * float(seq["n"][i])
+    return owner, norm
+
+
+def loss_coefficients(weight, adv, mask, seq_offsets, seq, grp, batch, params: Params):
+    """Per-token factor w_t A_i / norm_t that multiplies grad r_t in Eq. ACRL
+    (0 on masked tokens)."""
+    w = np.asarray(weight, dtype=np.float64)
+    A = np.asarray(adv, dtype=np.float64)
+    T = len(w)
+    m = np.ones(T, dtype=bool) if mask is None else (np.asarray(mask) != 0)
+    owner, norm = _norms(mask, seq_offsets, seq, grp, batch, params)
+    coef = np.zeros(T)
+    for t in range(T):
+        if m[t] and owner[t] >= 0 and norm[t] > 0:
+            coef[t] = w[t] * A[owner[t]] / norm[t]
+    return coef
+
+
+def surrogate_loss(logp, old_logp, adv, weight, mask, seq_offsets, seq, grp, batch, params: Params):
+    """Token losses -w_t min(r A, clip(r) A) / norm_t of Eq. ACRL from the
+    current log-probs alone (r = exp(logp - old_logp), or 1 without old_logp).
+    Returns (token_loss [T], total)."""
+    w = np.asarray(weight, dtype=np.float64)
+    A = np.asarray(adv, dtype=np.float64)
+    T = len(w)
+    m = np.ones(T, dtype=bool) if mask is None else (np.asarray(mask) != 0)
+    owner, norm = _norms(mask, seq_offsets, seq, grp, batch, params)
+    eps = params.clip_eps
+    tl = np.zeros(T)
+    for t in range(T):
+        i = owner[t]
+        if not m[t] or i < 0 or norm[t] <= 0:
+            continue
+        r = 1.0 if old_logp is None else math.exp(float(logp[t]) - float(old_logp[t]))
+        rc = min(max(r, 1.0 - eps), 1.0 + eps)
+        tl[t] = -w[t] * min(r * A[i], rc * A[i]) / norm[t]
+    return tl, math.fsum(tl)
+
+
 # --------------------------------------------------------------------------
 # whole step (for tests and the CPU baseline)
 # --------------------------------------------------------------------------

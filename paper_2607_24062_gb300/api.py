@@ -1,0 +1,218 @@
+"""Python binding of the ACRL C ABI: one function per entry point, same names
+without the `acrl_` prefix.  Arguments are torch tensors on the current CUDA
+device; this layer only checks dtypes/shapes, passes raw pointers and the
+current stream, allocates outputs the caller did not provide, and turns a
+non-OK status into an exception.  Every step of the computation runs in the
+library's kernels."""
+
+from __future__ import annotations
+
+import ctypes
+from dataclasses import dataclass
+
+import numpy as np
+import torch
+
+from . import _abi
+from ._abi import BATCH_DTYPE, GRP_DTYPE, SEQ_DTYPE, STATE_DTYPE, AcrlError, Params, check, lib
+
+
+def _ptr(t: torch.Tensor | None) -> int | None:
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+def _need(t: torch.Tensor, dtype, n: int | None, name: str):
+    if not isinstance(t, torch.Tensor):
+        raise AcrlError(f"{name}: expected a torch tensor")
+    if t.dtype != dtype:
+        raise AcrlError(f"{name}: dtype {t.dtype}, expected {dtype}")
+    if not t.is_cuda:
+        raise AcrlError(f"{name}: must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise AcrlError(f"{name}: must be contiguous")
+    if n is not None and t.numel() < n:
+        raise AcrlError(f"{name}: has {t.numel()} elements, needs {n}")
+    return t
+
+
+def _opt(t, dtype, n, name):
+    return None if t is None else _need(t, dtype, n, name)
+
+
+def _rows(x: torch.Tensor, name: str):
+    if x.dtype != torch.bfloat16 or x.dim() != 2:
+        raise AcrlError(f"{name}: expected a 2-D bfloat16 tensor")
+    if not x.is_cuda or x.stride(1) != 1:
+        raise AcrlError(f"{name}: must be a CUDA tensor with unit column stride")
+    return x.shape[0], x.stride(0)
+
+
+def struct_buffer(dtype: np.dtype, n: int, device=None) -> torch.Tensor:
+    """Device bytes for n ABI structs."""
+    return torch.zeros(max(1, n) * dtype.itemsize, dtype=torch.uint8, device=device or "cuda")
+
+
+def read_structs(buf: torch.Tensor, dtype: np.dtype, n: int) -> np.ndarray:
+    return buf[: n * dtype.itemsize].cpu().numpy().view(dtype)
+
+
+def new_flags(device=None) -> torch.Tensor:
+    return torch.zeros(1, dtype=torch.int32, device=device or "cuda")
+
+
+def token_stats(logits, ids, mask=None, *, V=None, lse=None, logp=None, entropy=None, flags=None, stream=None):
+    """acrl_token_stats.  Returns (lse, logp, entropy) float32 [T]."""
+    T, ld = _rows(logits, "logits")
+    V = ld if V is None else V
+    dev = logits.device
+    _need(ids, torch.int32, T, "ids")
+    _opt(mask, torch.uint8, T, "mask")
+    lse = torch.empty(T, dtype=torch.float32, device=dev) if lse is None else _need(lse, torch.float32, T, "lse")
+    logp = torch.empty(T, dtype=torch.float32, device=dev) if logp is None else _need(logp, torch.float32, T, "logp")
+    entropy = torch.empty(T, dtype=torch.float32, device=dev) if entropy is None else \
+        _need(entropy, torch.float32, T, "entropy")
+    flags = new_flags(dev) if flags is None else flags
+    check(lib().acrl_token_stats(_ptr(logits), T, V, ld, _ptr(ids), _ptr(mask), _ptr(lse), _ptr(logp),
+                                 _ptr(entropy), _ptr(flags), _stream(stream)), "acrl_token_stats")
+    return lse, logp, entropy
+
+
+@dataclass
+class Discrepancy:
+    lr: torch.Tensor
+    d: torch.Tensor
+    seq: torch.Tensor    # device bytes of acrl_seq_stats[S]
+    grp: torch.Tensor    # device bytes of acrl_group_stats[Gn]
+    batch: torch.Tensor  # device bytes of acrl_batch_stats
+    S: int
+    Gn: int
+
+    def seq_host(self):
+        return read_structs(self.seq, SEQ_DTYPE, self.S)
+
+    def grp_host(self):
+        return read_structs(self.grp, GRP_DTYPE, self.Gn)
+
+    def batch_host(self):
+        return read_structs(self.batch, BATCH_DTYPE, 1)[0]
+
+
+def seq_discrepancy(logp_pi, logp_mu, mask, seq_offsets, group_offsets, entropy=None, *, out: Discrepancy | None = None,
+                    flags=None, stream=None) -> Discrepancy:
+    """acrl_seq_discrepancy."""
+    T = logp_pi.numel()
+    S = seq_offsets.numel() - 1
+    Gn = group_offsets.numel() - 1
+    dev = logp_pi.device
+    _need(logp_pi, torch.float32, T, "logp_pi")
+    _need(logp_mu, torch.float32, T, "logp_mu")
+    _opt(mask, torch.uint8, T, "mask")
+    _need(seq_offsets, torch.int64, S + 1, "seq_offsets")
+    _need(group_offsets, torch.int32, Gn + 1, "group_offsets")
+    _opt(entropy, torch.float32, T, "entropy")
+    if out is None:
+        out = Discrepancy(torch.empty(T, dtype=torch.float32, device=dev), torch.empty(T, dtype=torch.float32, device=dev),
+                          struct_buffer(SEQ_DTYPE, S, dev), struct_buffer(GRP_DTYPE, Gn, dev),
+                          struct_buffer(BATCH_DTYPE, 1, dev), S, Gn)
+    flags = new_flags(dev) if flags is None else flags
+    check(lib().acrl_seq_discrepancy(_ptr(logp_pi), _ptr(logp_mu), _ptr(mask), T, _ptr(seq_offsets), S,
+                                     _ptr(group_offsets), Gn, _ptr(entropy), _ptr(out.lr), _ptr(out.d), _ptr(out.seq),
+                                     _ptr(out.grp), _ptr(out.batch), _ptr(flags), _stream(stream)),
+          "acrl_seq_discrepancy")
+    return out
+
+
+def grpo_advantage(rewards, group_offsets, params: Params, *, adv=None, flags=None, stream=None):
+    """acrl_grpo_advantage.  Returns adv float32 [S]."""
+    S = rewards.numel()
+    Gn = group_offsets.numel() - 1
+    _need(rewards, torch.float32, S, "rewards")
+    _need(group_offsets, torch.int32, Gn + 1, "group_offsets")
+    adv = torch.empty(S, dtype=torch.float32, device=rewards.device) if adv is None else _need(adv, torch.float32, S, "adv")
+    flags = new_flags(rewards.device) if flags is None else flags
+    check(lib().acrl_grpo_advantage(_ptr(rewards), _ptr(group_offsets), Gn, S, ctypes.byref(params), _ptr(adv),
+                                    _ptr(flags), _stream(stream)), "acrl_grpo_advantage")
+    return adv
+
+
+def controller_init(params: Params, state=None, device=None, stream=None) -> torch.Tensor:
+    """acrl_controller_init; allocates the 48-byte device state if not given."""
+    state = struct_buffer(STATE_DTYPE, 1, device) if state is None else state
+    check(lib().acrl_controller_init(_ptr(state), ctypes.byref(params), _stream(stream)), "acrl_controller_init")
+    return state
+
+
+def read_state(state: torch.Tensor) -> np.void:
+    return read_structs(state, STATE_DTYPE, 1)[0]
+
+
+def controller_step(state, params: Params, disc: Discrepancy, mask, seq_offsets, group_offsets, adv, *, weight=None,
+                    coef=None, alpha=None, flags=None, stream=None):
+    """acrl_controller_step.  Returns (weight [T], coef [T], alpha [S])."""
+    T = disc.lr.numel()
+    dev = disc.lr.device
+    weight = torch.empty(T, dtype=torch.float32, device=dev) if weight is None else _need(weight, torch.float32, T, "weight")
+    coef = torch.empty(T, dtype=torch.float32, device=dev) if coef is None else _need(coef, torch.float32, T, "coef")
+    alpha = torch.empty(disc.S, dtype=torch.float32, device=dev) if alpha is None else \
+        _need(alpha, torch.float32, disc.S, "alpha")
+    _need(adv, torch.float32, disc.S, "adv")
+    _opt(mask, torch.uint8, T, "mask")
+    flags = new_flags(dev) if flags is None else flags
+    check(lib().acrl_controller_step(_ptr(state), ctypes.byref(params), _ptr(disc.lr), _ptr(mask), T,
+                                     _ptr(seq_offsets), disc.S, _ptr(group_offsets), disc.Gn, _ptr(disc.seq),
+                                     _ptr(disc.grp), _ptr(disc.batch), _ptr(adv), _ptr(weight), _ptr(coef),
+                                     _ptr(alpha), _ptr(flags), _stream(stream)), "acrl_controller_step")
+    return weight, coef, alpha
+
+
+def loss_grad_logits(logits, ids, mask, lse, old_logp, coef, clip_eps: float, *, V=None, grad=None, token_loss=None,
+                     loss=None, flags=None, stream=None):
+    """acrl_loss_grad_logits.  Returns (grad bf16 [T, ld], token_loss [T], loss [1])."""
+    T, ld = _rows(logits, "logits")
+    V = ld if V is None else V
+    dev = logits.device
+    _need(ids, torch.int32, T, "ids")
+    _opt(mask, torch.uint8, T, "mask")
+    _opt(lse, torch.float32, T, "lse")
+    _opt(old_logp, torch.float32, T, "old_logp")
+    _need(coef, torch.float32, T, "coef")
+    if grad is None:
+        grad = torch.empty((T, ld), dtype=torch.bfloat16, device=dev)
+    elif grad.dtype != torch.bfloat16 or grad.dim() != 2 or grad.stride(0) != ld or grad.stride(1) != 1 or \
+            grad.shape[0] < T:
+        raise AcrlError("grad: expected a bf16 [T, ld] tensor with the logits' row stride")
+    token_loss = torch.empty(T, dtype=torch.float32, device=dev) if token_loss is None else \
+        _need(token_loss, torch.float32, T, "token_loss")
+    loss = torch.empty(1, dtype=torch.float32, device=dev) if loss is None else _need(loss, torch.float32, 1, "loss")
+    flags = new_flags(dev) if flags is None else flags
+    check(lib().acrl_loss_grad_logits(_ptr(logits), T, V, ld, _ptr(ids), _ptr(mask), _ptr(lse), _ptr(old_logp),
+                                      _ptr(coef), float(clip_eps), _ptr(grad), _ptr(token_loss), _ptr(loss),
+                                      _ptr(flags), _stream(stream)), "acrl_loss_grad_logits")
+    return grad, token_loss, loss
+
+
+def reduce_loss(token_loss, *, loss=None, stream=None):
+    """acrl_reduce_loss."""
+    T = token_loss.numel()
+    _need(token_loss, torch.float32, T, "token_loss")
+    loss = torch.empty(1, dtype=torch.float32, device=token_loss.device) if loss is None else loss
+    check(lib().acrl_reduce_loss(_ptr(token_loss), T, _ptr(loss), _stream(stream)), "acrl_reduce_loss")
+    return loss
+
+
+def read_flags(flags, stream=None) -> int:
+    """acrl_read_flags (synchronises the stream)."""
+    host = ctypes.c_int32(0)
+    check(lib().acrl_read_flags(_ptr(flags), ctypes.byref(host), _stream(stream)), "acrl_read_flags")
+    return int(host.value)
+
+
+__all__ = ["Params", "AcrlError", "token_stats", "seq_discrepancy", "grpo_advantage", "controller_init",
+           "controller_step", "loss_grad_logits", "reduce_loss", "read_flags", "read_state", "Discrepancy",
+           "struct_buffer", "read_structs", "new_flags", "_abi"]

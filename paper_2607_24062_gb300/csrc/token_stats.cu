@@ -1,0 +1,129 @@
+// acrl_token_stats: one streaming pass over pi's bf16 logits per token row
+// giving the log-sum-exp, the sampled token's log-prob and the entropy.
+//
+// Each row is read exactly once from HBM with 16-byte non-allocating loads.
+// A team of threads (a warp for short rows, the whole CTA for vocabulary-size
+// rows) owns a row; every thread keeps an online base-2 state
+// (max, sum 2^(u-U), sum 2^(u-U)(u-U)) over its strided share of the row, and
+// the team merges the states with a fixed butterfly/tree order, so results
+// are bit-reproducible run to run.
+#include "acrl_device.cuh"
+#include "acrl_host.h"
+#include "row_lse.cuh"
+
+namespace acrl {
+namespace {
+
+// Outputs of one row from its merged state; mx is the row maximum (natural units).
+__device__ __forceinline__ void row_outputs(const LseAcc& acc, float mx, const acrl_bf16* row, int V, int a,
+                                            float* lse, float* logp, float* ent, int64_t t, int32_t* flags) {
+    const float l2s0 = log2f(acc.s0);
+    // acc.U is mx*log2(e) rounded; c is that rounding error, exact through the FMA
+    const float c = fmaf(mx, kLog2e, -acc.U);
+    const float lse_v = fmaf(kLn2, l2s0 - c, mx);
+    const float H = kLn2 * (l2s0 - acc.s1 / acc.s0);
+    float lp = 0.f;
+    if (a >= 0 && a < V) {
+        lp = (bf16_to_float(row[a]) - mx) - kLn2 * (l2s0 - c);
+    } else {
+        raise_flag(flags, ACRL_FLAG_BAD_ID);
+    }
+    if (!isfinite(lse_v) || !isfinite(H)) {
+        raise_flag(flags, ACRL_FLAG_NONFINITE);
+        lse[t] = logp[t] = ent[t] = __int_as_float(0x7fc00000);
+        return;
+    }
+    lse[t] = lse_v;
+    logp[t] = lp;
+    ent[t] = H;
+}
+
+// A whole CTA per row (vocabulary-size rows).
+template <int THREADS, int UNROLL>
+__global__ void __launch_bounds__(THREADS) token_stats_cta(const acrl_bf16* __restrict__ logits, int64_t T, int V,
+                                                           int64_t ld, const int32_t* __restrict__ ids,
+                                                           const uint8_t* __restrict__ mask, float* __restrict__ lse,
+                                                           float* __restrict__ logp, float* __restrict__ ent,
+                                                           int32_t* flags) {
+    constexpr int NW = THREADS / 32;
+    __shared__ LseAcc part[NW];
+    __shared__ float pmax[NW];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    for (int64_t t = blockIdx.x; t < T; t += gridDim.x) {
+        if (mask && mask[t] == 0) {
+            if (threadIdx.x == 0) lse[t] = logp[t] = ent[t] = 0.f;
+            continue;
+        }
+        const acrl_bf16* row = logits + t * ld;
+        float mx;
+        LseAcc acc = row_partial<THREADS, UNROLL>(row, V, threadIdx.x, mx);
+        acc = warp_lse(acc);
+        mx = warp_max(mx);
+        if (lane == 0) {
+            part[wid] = acc;
+            pmax[wid] = mx;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            LseAcc r = part[0];
+            float m = pmax[0];
+#pragma unroll
+            for (int w = 1; w < NW; ++w) {
+                r = lse_merge(r, part[w]);
+                m = fmaxf(m, pmax[w]);
+            }
+            row_outputs(r, m, row, V, ids[t], lse, logp, ent, t, flags);
+        }
+        __syncthreads();
+    }
+}
+
+// One warp per row (short rows); THREADS/32 rows per CTA.
+template <int THREADS, int UNROLL>
+__global__ void __launch_bounds__(THREADS) token_stats_warp(const acrl_bf16* __restrict__ logits, int64_t T, int V,
+                                                            int64_t ld, const int32_t* __restrict__ ids,
+                                                            const uint8_t* __restrict__ mask, float* __restrict__ lse,
+                                                            float* __restrict__ logp, float* __restrict__ ent,
+                                                            int32_t* flags) {
+    constexpr int NW = THREADS / 32;
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    for (int64_t t = int64_t(blockIdx.x) * NW + wid; t < T; t += int64_t(gridDim.x) * NW) {
+        if (mask && mask[t] == 0) {
+            if (lane == 0) lse[t] = logp[t] = ent[t] = 0.f;
+            continue;
+        }
+        const acrl_bf16* row = logits + t * ld;
+        float mx;
+        LseAcc acc = row_partial<32, UNROLL>(row, V, lane, mx);
+        acc = warp_lse(acc);
+        mx = warp_max(mx);
+        if (lane == 0) row_outputs(acc, mx, row, V, ids[t], lse, logp, ent, t, flags);
+    }
+}
+
+}  // namespace
+
+}  // namespace acrl
+
+using namespace acrl;
+
+extern "C" acrl_status acrl_token_stats(const acrl_bf16* logits, int64_t T, int64_t V, int64_t ld,
+                                        const int32_t* ids, const uint8_t* mask, float* lse, float* logp,
+                                        float* entropy, int32_t* dev_flags, acrl_stream stream) {
+    if (T < 0 || V < 1 || V > kMaxVocab || ld < V || (ld & 7) != 0) return ACRL_ERR_INVALID_ARG;
+    if (T == 0) return ACRL_OK;
+    if (!logits || !ids || !lse || !logp || !entropy || !dev_flags) return ACRL_ERR_INVALID_ARG;
+    if (!aligned16(logits)) return ACRL_ERR_INVALID_ARG;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const int v = int(V);
+    if (V <= kWarpRowMaxV) {
+        constexpr int THREADS = 256;
+        token_stats_warp<THREADS, 4><<<unsigned(grid_for(THREADS / 32, T)), THREADS, 0, s>>>(
+            logits, T, v, ld, ids, mask, lse, logp, entropy, dev_flags);
+    } else {
+        constexpr int THREADS = 512;
+        token_stats_cta<THREADS, 4><<<unsigned(grid_for(1, T)), THREADS, 0, s>>>(
+            logits, T, v, ld, ids, mask, lse, logp, entropy, dev_flags);
+    }
+    return launch_status();
+}

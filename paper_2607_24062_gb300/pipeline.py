@@ -1,0 +1,107 @@
+"""One on-policy ACRL pass over a batch: the five C-ABI calls in order on one
+stream, with every buffer allocated once per batch shape.
+
+    token_stats -> seq_discrepancy -> grpo_advantage -> controller_step
+                -> loss_grad_logits
+
+The weights need Y_g, which needs every row of the prompt, so the gradient
+pass can only start after the statistics pass has seen the whole batch: the
+logits are streamed twice (2 + 4 bytes per element).  For batches whose
+gradient does not fit beside the logits, `run(..., chunk_rows=k)` runs the
+gradient pass k rows at a time into a chunk-sized buffer and hands each chunk
+to a callback.
+"""
+
+from __future__ import annotations
+
+from typing import Callable
+
+import torch
+
+from . import api
+from ._abi import BATCH_DTYPE, GRP_DTYPE, SEQ_DTYPE, Params
+
+
+class AcrlStep:
+    def __init__(self, T: int, V: int, ld: int, S: int, Gn: int, params: Params, device="cuda",
+                 grad_rows: int | None = None):
+        dev = torch.device(device)
+        f32 = dict(dtype=torch.float32, device=dev)
+        self.T, self.V, self.ld, self.S, self.Gn = T, V, ld, S, Gn
+        self.params = params
+        self.lse = torch.empty(T, **f32)
+        self.logp = torch.empty(T, **f32)
+        self.entropy = torch.empty(T, **f32)
+        self.disc = api.Discrepancy(torch.empty(T, **f32), torch.empty(T, **f32),
+                                    api.struct_buffer(SEQ_DTYPE, S, dev), api.struct_buffer(GRP_DTYPE, Gn, dev),
+                                    api.struct_buffer(BATCH_DTYPE, 1, dev), S, Gn)
+        self.adv = torch.empty(S, **f32)
+        self.weight = torch.empty(T, **f32)
+        self.coef = torch.empty(T, **f32)
+        self.alpha = torch.empty(S, **f32)
+        self.grad = torch.empty((grad_rows if grad_rows else T, ld), dtype=torch.bfloat16, device=dev)
+        self.token_loss = torch.empty(T, **f32)
+        self.loss = torch.empty(1, **f32)
+        self.chunk_loss = torch.empty(1, **f32)
+        self.flags = api.new_flags(dev)
+        self.state = api.controller_init(params, device=dev)
+
+    def reset_controller(self, stream=None):
+        api.controller_init(self.params, state=self.state, stream=stream)
+
+    def statistics(self, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, stream=None):
+        """Everything up to and including the controller (one read of the logits)."""
+        p = self.params
+        api.token_stats(logits, ids, mask, V=self.V, lse=self.lse, logp=self.logp, entropy=self.entropy,
+                        flags=self.flags, stream=stream)
+        api.seq_discrepancy(self.logp, logp_mu, mask, seq_offsets, group_offsets, self.entropy, out=self.disc,
+                            flags=self.flags, stream=stream)
+        api.grpo_advantage(rewards, group_offsets, p, adv=self.adv, flags=self.flags, stream=stream)
+        api.controller_step(self.state, p, self.disc, mask, seq_offsets, group_offsets, self.adv,
+                            weight=self.weight, coef=self.coef, alpha=self.alpha, flags=self.flags, stream=stream)
+
+    def gradient(self, logits, ids, mask, stream=None, old_logp=None, recompute_lse=False,
+                 chunk_rows: int | None = None, on_chunk: Callable[[int, int, torch.Tensor], None] | None = None):
+        """The loss and dL/dlogits (second read of the logits, one write)."""
+        lse = None if recompute_lse else self.lse
+        eps = self.params.clip_eps
+        if not chunk_rows:
+            api.loss_grad_logits(logits, ids, mask, lse, old_logp, self.coef, eps, V=self.V, grad=self.grad,
+                                 token_loss=self.token_loss, loss=self.loss, flags=self.flags, stream=stream)
+            return
+        for r0 in range(0, self.T, chunk_rows):
+            r1 = min(self.T, r0 + chunk_rows)
+            g = self.grad[: r1 - r0]
+            api.loss_grad_logits(logits[r0:r1], ids[r0:r1], None if mask is None else mask[r0:r1],
+                                 None if lse is None else lse[r0:r1],
+                                 None if old_logp is None else old_logp[r0:r1], self.coef[r0:r1], eps, V=self.V,
+                                 grad=g, token_loss=self.token_loss[r0:r1], loss=self.chunk_loss, flags=self.flags,
+                                 stream=stream)
+            if on_chunk is not None:
+                on_chunk(r0, r1, g)
+        api.reduce_loss(self.token_loss, loss=self.loss, stream=stream)
+
+    def run(self, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, stream=None, **grad_kw):
+        self.statistics(logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, stream=stream)
+        self.gradient(logits, ids, mask, stream=stream, **grad_kw)
+
+    @classmethod
+    def for_batch(cls, batch, params: Params, device="cuda", grad_rows=None):
+        return cls(batch.T, batch.V, batch.ld, batch.S, batch.Gn, params, device=device, grad_rows=grad_rows)
+
+    def run_batch(self, batch, stream=None, **grad_kw):
+        self.run(batch.logits, batch.ids, batch.mask, batch.logp_mu, batch.rewards, batch.seq_offsets,
+                 batch.group_offsets, stream=stream, **grad_kw)
+
+    # host views -----------------------------------------------------------
+    def seq_host(self):
+        return self.disc.seq_host()
+
+    def grp_host(self):
+        return self.disc.grp_host()
+
+    def batch_host(self):
+        return self.disc.batch_host()
+
+    def state_host(self):
+        return api.read_state(self.state)

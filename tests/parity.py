@@ -1,0 +1,113 @@
+"""Helpers for comparing the CUDA path (through the C ABI) with the float64
+oracle on the same seeded inputs.  Tolerances are the ones the method's
+arithmetic supports (bf16 in, fp32 accumulation):
+  * log-probs / lse: 2e-4 absolute;
+  * entropy, weights, alpha, aggregates, X, batch statistics, loss: 1e-3
+    relative (entropy with a 1e-5 absolute floor);
+  * bf16 gradient elements: 1e-2 relative; an element whose reference is
+    below 2^-125 may come back as 0 (the exp2 flushes subnormals); the
+    sampled column, coef * (p_a - 1), carries the fp32 error of logp_a, so it
+    also gets an absolute floor of 1e-5 * |coef|.
+Integer outputs (counts, group indices, flags) must match exactly."""
+
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle as O
+
+TOL_LOGP = 2e-4
+TOL_REL = 1e-3
+TOL_GRAD = 1e-2
+FTZ = 2.0 ** -125
+
+
+def host(t):
+    return t.detach().cpu().numpy()
+
+
+def oracle_params(p) -> O.Params:
+    return O.Params(gamma=float(p.gamma), C=float(p.C), clip_eps=float(p.clip_eps), adv_eps=float(p.adv_eps),
+                    mode=int(p.mode), y_gran=int(p.y_gran), agg=int(p.agg), adv_ddof=int(p.adv_ddof),
+                    singleton_rule=int(p.singleton_rule), calib_steps=int(p.calib_steps), X_init=float(p.X_init))
+
+
+def rows_f64(logits: torch.Tensor, rows, V: int) -> np.ndarray:
+    """Exact float64 copy of the bf16 logits of `rows` (first V columns)."""
+    idx = torch.as_tensor(np.asarray(rows, dtype=np.int64), device=logits.device)
+    bits = logits.index_select(0, idx)[:, :V].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    return O.bf16_bits_to_f64(bits)
+
+
+def grad_rows(grad: torch.Tensor, rows, V: int) -> np.ndarray:
+    idx = torch.as_tensor(np.asarray(rows, dtype=np.int64), device=grad.device)
+    return grad.index_select(0, idx)[:, :V].float().cpu().numpy().astype(np.float64)
+
+
+def assert_close_rel(got, ref, rel=TOL_REL, floor=0.0, what=""):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    bad = np.abs(got - ref) > rel * np.abs(ref) + floor
+    bad &= ~(np.isnan(got) & np.isnan(ref))
+    if bad.any():
+        k = np.flatnonzero(bad.ravel())[:5]
+        raise AssertionError(f"{what}: {bad.sum()} of {bad.size} outside rel {rel} floor {floor}; "
+                             f"got {got.ravel()[k]} ref {ref.ravel()[k]} at {k}")
+
+
+def assert_close_abs(got, ref, tol, what=""):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    bad = np.abs(got - ref) > tol
+    bad &= ~(np.isnan(got) & np.isnan(ref))
+    if bad.any():
+        k = np.flatnonzero(bad.ravel())[:5]
+        raise AssertionError(f"{what}: {bad.sum()} of {bad.size} outside abs {tol}; got {got.ravel()[k]} "
+                             f"ref {ref.ravel()[k]} at {k}")
+
+
+def assert_grad_rows(got, ref, coef_eff, ids_rows, what="grad"):
+    """got/ref [R, V]; coef_eff [R] = the reference coef_t g_t r_t."""
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    tol = TOL_GRAD * np.abs(ref)
+    tol = np.maximum(tol, np.where(np.abs(ref) < FTZ, FTZ, 0.0))
+    R = ref.shape[0]
+    cols = np.asarray(ids_rows, dtype=np.int64)
+    ok_ids = (cols >= 0) & (cols < ref.shape[1])
+    r_idx = np.arange(R)[ok_ids]
+    tol[r_idx, cols[ok_ids]] += 1e-5 * np.abs(np.asarray(coef_eff)[ok_ids])
+    bad = np.abs(got - ref) > tol
+    if bad.any():
+        rr, cc = np.nonzero(bad)
+        raise AssertionError(f"{what}: {bad.sum()} of {bad.size} elements off; first rows {rr[:5]} cols {cc[:5]} "
+                             f"got {got[rr[:5], cc[:5]]} ref {ref[rr[:5], cc[:5]]}")
+
+
+def compare_seq(gpu_seq, ref_seq, what="seq"):
+    assert np.array_equal(gpu_seq["n"], ref_seq["n"]), f"{what}.n"
+    assert np.array_equal(gpu_seq["group"], ref_seq["group"]), f"{what}.group"
+    assert_close_rel(gpu_seq["mean_d"], ref_seq["mean_d"], floor=1e-7, what=f"{what}.mean_d")
+    assert_close_rel(gpu_seq["max_d"], ref_seq["max_d"], floor=1e-7, what=f"{what}.max_d")
+    assert_close_rel(gpu_seq["sum_d"], ref_seq["sum_d"], floor=1e-6, what=f"{what}.sum_d")
+    assert_close_rel(gpu_seq["sum_d2"], ref_seq["sum_d2"], floor=1e-7, what=f"{what}.sum_d2")
+    # S_i = log rho_i: an absolute quantity; its exp is the MIS weight
+    assert_close_abs(gpu_seq["sum_lr"], ref_seq["sum_lr"], TOL_REL * np.maximum(1.0, np.abs(ref_seq["sum_lr"])),
+                     what=f"{what}.sum_lr")
+
+
+def compare_grp(gpu_grp, ref_grp, what="grp"):
+    assert np.array_equal(gpu_grp["n_valid_seqs"], ref_grp["n_valid_seqs"]), f"{what}.n_valid_seqs"
+    assert np.array_equal(gpu_grp["n_tokens"], ref_grp["n_tokens"]), f"{what}.n_tokens"
+    assert_close_rel(gpu_grp["Y"], ref_grp["Y"], floor=1e-9, what=f"{what}.Y")
+
+
+def compare_batch(gb, rb, what="batch"):
+    assert int(gb["n_tokens"]) == rb["n_tokens"], f"{what}.n_tokens"
+    assert int(gb["n_groups_valid"]) == rb["n_groups_valid"], f"{what}.n_groups_valid"
+    assert int(gb["n_seqs_valid"]) == rb["n_seqs_valid"], f"{what}.n_seqs_valid"
+    for k in ("d_mean", "d_max", "d_std", "Y_sum", "Y_mean"):
+        assert_close_rel(gb[k], rb[k], floor=1e-9, what=f"{what}.{k}")
+    assert_close_rel(gb["H_mean"], rb["H_mean"], floor=1e-5, what=f"{what}.H_mean")
+    assert_close_abs(gb["lr_mean"], rb["lr_mean"], TOL_LOGP, what=f"{what}.lr_mean")

@@ -1,0 +1,72 @@
+"""The C-ABI library builds for sm_103a, loads, exports every function that
+include/acrl.h declares, agrees with the binding on struct layouts, and
+rejects bad host-side arguments before touching a GPU.  CPU only: no call
+here launches a kernel."""
+
+import ctypes
+import shutil
+
+import pytest
+
+from paper_2607_24062_gb300 import _abi, build
+
+pytestmark = pytest.mark.skipif(shutil.which("nvcc") is None and not build.up_to_date(),
+                                reason="needs nvcc to build the library")
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    return _abi.lib()
+
+
+def test_exports_every_declared_function(L):
+    declared = _abi.header_functions()
+    assert len(declared) >= 11
+    for name in declared:
+        assert hasattr(L, name), name
+    assert set(declared) == set(_abi.SIGNATURES)
+
+
+def test_abi_version_and_layouts(L):
+    assert L.acrl_abi_version() == 1
+    assert L.acrl_struct_size(0) == ctypes.sizeof(_abi.Params) == 48
+    assert L.acrl_struct_size(1) == 48 and L.acrl_struct_size(2) == 64
+    assert L.acrl_struct_size(3) == 24 and L.acrl_struct_size(4) == 104
+    assert L.acrl_struct_size(99) == -1
+    assert L.acrl_status_string(0) == b"ok" and L.acrl_status_string(1) == b"invalid argument"
+
+
+def test_host_side_rejections(L):
+    p = _abi.Params()
+    bad = _abi.Params(C=1.0)
+    E = _abi.ERR_INVALID_ARG
+    fake = 0x1000  # never dereferenced: every call below is rejected on the host
+    # token stats: ld < V, ld not a multiple of 8, misaligned logits, null outputs
+    assert L.acrl_token_stats(fake, 4, 16, 8, fake, None, fake, fake, fake, fake, None) == E
+    assert L.acrl_token_stats(fake, 4, 16, 20, fake, None, fake, fake, fake, fake, None) == E
+    assert L.acrl_token_stats(fake + 2, 4, 16, 16, fake, None, fake, fake, fake, fake, None) == E
+    assert L.acrl_token_stats(fake, 4, 16, 16, fake, None, None, fake, fake, fake, None) == E
+    assert L.acrl_token_stats(fake, -1, 16, 16, fake, None, fake, fake, fake, fake, None) == E
+    # T = 0 is a valid no-op
+    assert L.acrl_token_stats(None, 0, 16, 16, None, None, None, None, None, None, None) == _abi.OK
+    # hyper-parameters out of range
+    assert L.acrl_grpo_advantage(fake, fake, 1, 1, ctypes.byref(bad), fake, fake, None) == E
+    assert L.acrl_controller_init(None, ctypes.byref(p), None) == E
+    assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(gamma=0.0)), None) == E
+    assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(calib_steps=0)), None) == E
+    assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(mode=7)), None) == E
+    # loss/grad: clip eps out of range, misaligned grad
+    assert L.acrl_loss_grad_logits(fake, 4, 16, 16, fake, None, None, None, fake, 1.5, fake, fake, fake, fake,
+                                   None) == E
+    assert L.acrl_loss_grad_logits(fake, 4, 16, 16, fake, None, None, None, fake, 0.2, fake + 8, fake, fake, fake,
+                                   None) == E
+    assert L.acrl_read_flags(None, None, None) == E
+    assert L.acrl_reduce_loss(None, 4, fake, None) == E
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(_abi, "LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(_abi, "_LIB", None)
+    with pytest.raises(_abi.AcrlError):
+        _abi.lib()

@@ -481,3 +481,26 @@ def test_full_step_mu_equals_pi_fixed_point():
     res = O.step(z, ids, None, logp, np.array([1.0, 0.0, 1.0]), [0, 4, 8, 12], [0, 3], O.Params())
     assert np.all(res.lr == 0) and np.all(res.weight == 1.0)
     assert res.state.X == 0.0 and res.flags & O.FLAG_X_NONPOS
+
+
+@pytest.mark.parametrize("with_old", [False, True])
+def test_coefficients_and_surrogate_agree_with_gradient(with_old):
+    # coef_t (p - onehot) r g must reproduce the autograd-pinned gradient, and the
+    # O(T) surrogate loss must equal the loss of loss_grad_logits.
+    rng = np.random.default_rng(44 + with_old)
+    f = _fixture(rng, with_old=with_old)
+    p = O.Params()
+    grad, tl, loss = O.loss_grad_logits(f["z"], f["ids"], f["mask"], None, f["old"], f["adv"], f["w"], f["so"],
+                                        f["seq"], f["grp"], f["batch"], p)
+    coef = O.loss_coefficients(f["w"], f["adv"], f["mask"], f["so"], f["seq"], f["grp"], f["batch"], p)
+    lse, logp, _, _ = O.token_stats(f["z"], f["ids"], f["mask"])
+    tl2, loss2 = O.surrogate_loss(logp, f["old"], f["adv"], f["w"], f["mask"], f["so"], f["seq"], f["grp"],
+                                  f["batch"], p)
+    assert loss2 == pytest.approx(loss, abs=1e-14)
+    np.testing.assert_allclose(tl2, tl, atol=1e-15)
+    for t in range(len(coef)):
+        r = 1.0 if f["old"] is None else math.exp(logp[t] - f["old"][t])
+        gate = (coef[t] >= 0 and r <= 1.2) or (coef[t] < 0 and r >= 0.8)
+        pr = np.exp(f["z"][t] - lse[t])
+        pr[f["ids"][t]] -= 1.0
+        np.testing.assert_allclose(grad[t], coef[t] * r * gate * pr, atol=1e-15)

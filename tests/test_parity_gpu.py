@@ -1,0 +1,355 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the float64
+oracle on the same seeded inputs.  Small shapes are compared element by
+element over the whole chain; the full-size workloads on sampled rows plus
+every O(T) output."""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import workloads as W
+from parity import (TOL_LOGP, assert_close_abs, assert_close_rel, assert_grad_rows, compare_batch, compare_grp,
+                    compare_seq, grad_rows, host, oracle_params, rows_f64)
+
+pytestmark = pytest.mark.gpu
+
+import paper_2607_24062_gb300 as acrl  # noqa: E402
+from paper_2607_24062_gb300 import api  # noqa: E402
+
+DEV = "cuda"
+
+
+def _gen(spec, seed=None, mutate=None):
+    b = W.generate(spec, seed=seed, device=DEV)
+    if mutate:
+        mutate(b)
+    return b
+
+
+def _host_inputs(b):
+    return dict(ids=host(b.ids), mask=host(b.mask), mu=host(b.logp_mu).astype(np.float64),
+                R=host(b.rewards).astype(np.float64), so=host(b.seq_offsets), go=host(b.group_offsets))
+
+
+def _full_chain_check(b, params, state=None):
+    """Run the GPU step and the oracle step on every row; compare everything."""
+    step = acrl.AcrlStep.for_batch(b, params)
+    if state is not None:
+        step.state.copy_(state)
+    step.run_batch(b)
+    torch.cuda.synchronize()
+    h = _host_inputs(b)
+    op = oracle_params(params)
+    z = rows_f64(b.logits, np.arange(b.T), b.V)
+    ostate = None
+    if state is not None:
+        s = api.read_structs(state, api.STATE_DTYPE, 1)[0]
+        ostate = O.ControllerState(X=float(s["X"]), calib_sum=float(s["calib_sum"]),
+                                   calib_count=int(s["calib_count"]), calib_done_steps=int(s["calib_done"]),
+                                   step=int(s["step"]), calibrated=bool(s["calibrated"]))
+    res = O.step(z, h["ids"], h["mask"], h["mu"], h["R"], h["so"], h["go"], op, state=ostate)
+    # a1
+    assert_close_abs(host(step.logp), res.logp, TOL_LOGP, "logp")
+    assert_close_abs(host(step.lse), res.lse, TOL_LOGP, "lse")
+    assert_close_rel(host(step.entropy), res.H, floor=1e-5, what="entropy")
+    # a2/a3
+    assert_close_abs(host(step.disc.lr), res.lr, TOL_LOGP, "lr")
+    assert_close_rel(host(step.disc.d), res.d, floor=1e-7, what="d")
+    compare_seq(step.seq_host(), res.seq)
+    compare_grp(step.grp_host(), res.grp)
+    gb = step.batch_host()
+    compare_batch(gb, res.batch)
+    # a4
+    assert_close_rel(host(step.adv), res.adv, floor=1e-6, what="adv")
+    # a5
+    st = step.state_host()
+    assert bool(st["calibrated"]) == res.state.calibrated and int(st["step"]) == res.state.step
+    assert_close_rel(st["X"], res.state.X, floor=1e-12, what="X")
+    assert_close_rel(gb["X"], res.info["X"] if res.state.calibrated else 0.0, floor=1e-12, what="batch.X")
+    assert_close_rel(host(step.alpha), res.alpha, floor=1e-6, what="alpha")
+    assert_close_rel(host(step.weight), res.weight, floor=1e-7, what="weight")
+    assert_close_rel(gb["w_mean"], res.info["w_mean"], floor=1e-9, what="w_mean")
+    assert_close_rel(gb["trunc_frac"], res.info["trunc_frac"], floor=2.0 / max(1, res.batch["n_tokens"]),
+                     what="trunc_frac")
+    coef_ref = O.loss_coefficients(res.weight, res.adv, h["mask"], h["so"], res.seq, res.grp, res.batch, op)
+    assert_close_rel(host(step.coef), coef_ref, floor=1e-12, what="coef")
+    # a6
+    assert_close_rel(host(step.token_loss), res.token_loss, floor=1e-12, what="token_loss")
+    assert_close_rel(float(step.loss), res.loss, floor=1e-9, what="loss")
+    assert_grad_rows(grad_rows(step.grad, np.arange(b.T), b.V), res.grad, coef_ref, h["ids"])
+    flags = api.read_flags(step.flags)
+    assert flags == res.flags, (flags, res.flags)
+    return step, res
+
+
+SMALL = {
+    "tiny": W.TINY,
+    "ragged_warp": W.small_variant(W.GRPO, name="ragged_warp", n_prompts=3, group_size=4, len_lo=1, len_hi=90,
+                                   V=5003, pad_multiple=16, ld_pad=8),
+    "ragged_cta": W.small_variant(W.QWEN, name="ragged_cta", n_prompts=2, group_size=3, len_lo=3, len_hi=40,
+                                  V=20011, ld_pad=24),
+    "qwen_vocab": W.small_variant(W.QWEN, name="qwen_vocab", n_prompts=2, group_size=4, len_lo=8, len_hi=24),
+}
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_full_chain_small(name):
+    _full_chain_check(_gen(SMALL[name], seed=123), acrl.Params())
+
+
+def _empty_seq(b):
+    # response 1 fully masked, and its prompt's other members keep going
+    so = host(b.seq_offsets)
+    b.mask[int(so[1]):int(so[2])] = 0
+
+
+def test_empty_sequence_and_group():
+    spec = W.small_variant(W.GRPO, name="empties", n_prompts=3, group_size=2, len_lo=5, len_hi=50, V=3001)
+
+    def mutate(b):
+        so = host(b.seq_offsets)
+        b.mask[int(so[1]):int(so[2])] = 0          # one empty response
+        b.mask[int(so[4]):int(so[6])] = 0          # a whole empty prompt
+
+    step, res = _full_chain_check(_gen(spec, seed=9, mutate=mutate), acrl.Params())
+    assert res.batch["n_groups_valid"] == 2
+
+
+@pytest.mark.parametrize("mode", [acrl.MODE_NONE, acrl.MODE_TIS, acrl.MODE_MIS, acrl.MODE_ACRL])
+@pytest.mark.parametrize("y_gran", [acrl.Y_GROUP, acrl.Y_SEQUENCE, acrl.Y_BATCH])
+def test_modes(mode, y_gran):
+    if mode != acrl.MODE_ACRL and y_gran != acrl.Y_GROUP:
+        pytest.skip("y granularity only matters for ACRL")
+    spec = W.small_variant(W.QWEN, name="modes", n_prompts=3, group_size=4, len_lo=4, len_hi=60, V=2048,
+                           perturb_frac=0.5, perturb_std=0.3)
+    _full_chain_check(_gen(spec, seed=77), acrl.Params(mode=mode, y_gran=y_gran, gamma=1.3, C=5.0))
+
+
+@pytest.mark.parametrize("kw", [dict(agg=acrl.AGG_TOKEN_MEAN), dict(adv_ddof=0), dict(X_init=0.013),
+                                dict(singleton_rule=acrl.SINGLETON_ZERO), dict(calib_steps=2)])
+def test_param_options(kw):
+    spec = W.small_variant(W.TINY, name="opts", n_prompts=3, group_size=2, len_lo=20, len_hi=70, V=1000)
+    _full_chain_check(_gen(spec, seed=5), acrl.Params(**kw))
+
+
+def test_singletons_tiny_grpo_rule():
+    # tiny workload: 4 prompts with one response each; A = R under MEAN0_STD1
+    step, res = _full_chain_check(_gen(W.TINY), acrl.Params())
+    np.testing.assert_array_equal(host(step.adv), host(W.generate(W.TINY, device="cpu").rewards))
+
+
+def test_uniform_logits_and_equal_policies():
+    # uniform logits: logp = -ln V and H = ln V; mu = pi: lr = d = 0, every weight 1, X -> 0 (flagged)
+    T, V = 12, 151936
+    logits = torch.full((T, V), 0.5, dtype=torch.bfloat16, device=DEV)
+    ids = torch.randint(0, V, (T,), dtype=torch.int32, device=DEV)
+    lse, logp, H = api.token_stats(logits, ids, None, V=V)
+    assert_close_abs(host(logp), -math.log(V), 1e-5, "uniform logp")
+    assert_close_rel(host(H), math.log(V), rel=1e-5, what="uniform entropy")
+    so = torch.tensor([0, 4, 8, 12], dtype=torch.int64, device=DEV)
+    go = torch.tensor([0, 2, 3], dtype=torch.int32, device=DEV)
+    p = acrl.Params()
+    flags = api.new_flags()
+    disc = api.seq_discrepancy(logp, logp.clone(), None, so, go, H, flags=flags)
+    adv = api.grpo_advantage(torch.tensor([1.0, 0.0, 1.0], device=DEV), go, p, flags=flags)
+    state = api.controller_init(p)
+    w, coef, alpha = api.controller_step(state, p, disc, None, so, go, adv, flags=flags)
+    assert torch.all(disc.lr == 0) and torch.all(disc.d == 0)
+    assert torch.all(w == 1.0) and torch.all(alpha == 0.0)
+    assert float(api.read_state(state)["X"]) == 0.0
+    assert api.read_flags(flags) == acrl.FLAG_X_NONPOS
+
+
+def test_old_logp_and_recomputed_lse():
+    """Cached-old path: weights from old log-probs, LSE recomputed in the gradient kernel, r != 1 with clipping."""
+    spec = W.small_variant(W.QWEN, name="offpolicy", n_prompts=2, group_size=4, len_lo=10, len_hi=80, V=20011)
+    b = _gen(spec, seed=31)
+    p = acrl.Params()
+    gen = torch.Generator(device=DEV).manual_seed(3)
+    lse, logp, H = api.token_stats(b.logits, b.ids, b.mask, V=b.V)
+    old = (logp + 0.3 * torch.randn(b.T, generator=gen, device=DEV)).clamp(max=0.0)
+    disc = api.seq_discrepancy(old, b.logp_mu, b.mask, b.seq_offsets, b.group_offsets, H)
+    adv = api.grpo_advantage(b.rewards, b.group_offsets, p)
+    state = api.controller_init(p)
+    w, coef, alpha = api.controller_step(state, p, disc, b.mask, b.seq_offsets, b.group_offsets, adv)
+    for recompute in (False, True):
+        grad, tl, loss = api.loss_grad_logits(b.logits, b.ids, b.mask, None if recompute else lse, old, coef,
+                                              p.clip_eps, V=b.V)
+        torch.cuda.synchronize()
+        h = _host_inputs(b)
+        op = oracle_params(p)
+        z = rows_f64(b.logits, np.arange(b.T), b.V)
+        olse, ologp, oH, _ = O.token_stats(z, h["ids"], h["mask"])
+        oold = host(old).astype(np.float64)
+        lr, d, seq, grp, batch, _ = O.seq_discrepancy(oold, h["mu"], h["mask"], h["so"], h["go"], oH)
+        oadv = O.grpo_advantage(h["R"], h["go"], op)
+        ow, oalpha, ost, info, _ = O.controller_step(O.controller_init(op), op, lr, h["mask"], h["so"], h["go"], seq,
+                                                     grp, batch, oadv)
+        assert_close_rel(host(w), ow, floor=1e-7, what="weight")
+        ograd, otl, oloss = O.loss_grad_logits(z, h["ids"], h["mask"], None, oold, oadv, ow, h["so"], seq, grp,
+                                               batch, op)
+        coef_ref = O.loss_coefficients(ow, oadv, h["mask"], h["so"], seq, grp, batch, op)
+        r = np.exp(ologp - oold)
+        gate = np.where(coef_ref >= 0, r <= 1 + op.clip_eps, r >= 1 - op.clip_eps)
+        assert 0 < gate.sum() < len(gate)   # both branches exercised
+        assert_grad_rows(grad_rows(grad, np.arange(b.T), b.V), ograd, coef_ref * r * gate, h["ids"])
+        assert_close_rel(host(tl), otl, floor=1e-12, what="token_loss")
+        assert_close_rel(float(loss), oloss, floor=1e-9, what="loss")
+
+
+def test_chunked_gradient_matches_whole():
+    spec = W.small_variant(W.GRPO, name="chunks", n_prompts=2, group_size=4, len_lo=30, len_hi=200, V=32000)
+    b = _gen(spec, seed=4)
+    p = acrl.Params()
+    whole = acrl.AcrlStep.for_batch(b, p)
+    whole.run_batch(b)
+    chunked = acrl.AcrlStep.for_batch(b, p, grad_rows=100)
+    got = torch.empty_like(whole.grad)
+
+    def keep(r0, r1, g):
+        got[r0:r1].copy_(g)
+    chunked.run_batch(b, chunk_rows=100, on_chunk=keep)
+    torch.cuda.synchronize()
+    assert torch.equal(got[:, :b.V].view(torch.int16), whole.grad[:, :b.V].view(torch.int16))
+    assert torch.equal(chunked.token_loss, whole.token_loss)
+    assert float(chunked.loss) == float(whole.loss)
+
+
+def test_bit_reproducible():
+    spec = W.small_variant(W.QWEN, name="repro", n_prompts=2, group_size=3, len_lo=40, len_hi=90)
+    b = _gen(spec, seed=8)
+    outs = []
+    for _ in range(2):
+        s = acrl.AcrlStep.for_batch(b, acrl.Params())
+        s.run_batch(b)
+        torch.cuda.synchronize()
+        outs.append((s.lse.clone(), s.entropy.clone(), s.weight.clone(), s.grad.clone(), s.loss.clone(),
+                     s.disc.batch.clone()))
+    for x, y in zip(*outs):
+        assert torch.equal(x.view(torch.uint8) if x.dtype != torch.uint8 else x,
+                           y.view(torch.uint8) if y.dtype != torch.uint8 else y)
+
+
+# --------------------------------------------------------------------------
+# edge cases and device flags
+# --------------------------------------------------------------------------
+
+def _tiny_manual(T, V, ld=None):
+    ld = ld or ((V + 7) // 8) * 8
+    gen = torch.Generator(device=DEV).manual_seed(T * 1000 + V)
+    logits = torch.zeros((T, ld), dtype=torch.bfloat16, device=DEV)
+    logits[:, :V] = (2 * torch.randn((T, V), generator=gen, device=DEV)).to(torch.bfloat16)
+    ids = torch.randint(0, V, (T,), generator=gen, device=DEV, dtype=torch.int32)
+    return logits, ids
+
+
+@pytest.mark.parametrize("V", [1, 3, 7, 8, 9, 33, 16385])
+def test_token_stats_odd_widths(V):
+    T = 37
+    logits, ids = _tiny_manual(T, V)
+    lse, logp, H = api.token_stats(logits, ids, None, V=V)
+    z = rows_f64(logits, np.arange(T), V)
+    olse, ologp, oH, _ = O.token_stats(z, host(ids), None)
+    assert_close_abs(host(logp), ologp, TOL_LOGP, "logp")
+    assert_close_abs(host(lse), olse, TOL_LOGP, "lse")
+    assert_close_rel(host(H), oH, floor=1e-5, what="H")
+
+
+def test_empty_batch():
+    logits = torch.zeros((0, 8), dtype=torch.bfloat16, device=DEV)
+    ids = torch.zeros(0, dtype=torch.int32, device=DEV)
+    lse, logp, H = api.token_stats(logits, ids, None, V=8)
+    assert lse.numel() == 0
+
+
+def test_bad_ids_nonfinite_and_masked_rows():
+    T, V = 6, 40
+    logits, ids = _tiny_manual(T, V)
+    ids[1] = V          # out of range
+    ids[2] = -1
+    logits[3, 5] = float("nan")
+    logits[4, 0] = float("-inf")
+    mask = torch.ones(T, dtype=torch.uint8, device=DEV)
+    mask[5] = 0
+    logits[5, :] = float("nan")     # masked: never read
+    flags = api.new_flags()
+    lse, logp, H = api.token_stats(logits, ids, mask, V=V, flags=flags)
+    f = api.read_flags(flags)
+    assert f == (acrl.FLAG_BAD_ID | acrl.FLAG_NONFINITE)
+    lp = host(logp)
+    assert lp[1] == 0.0 and lp[2] == 0.0 and np.isnan(lp[3]) and np.isnan(host(H)[4]) and lp[5] == 0.0
+    z = rows_f64(logits, np.arange(T), V)
+    olse, ologp, oH, of = O.token_stats(z, host(ids), host(mask))
+    assert of == f
+    assert_close_abs(host(lse)[[0, 1, 2, 5]], olse[[0, 1, 2, 5]], TOL_LOGP, "lse")
+    # the gradient kernel zeroes rows it cannot use and raises BAD_ID too
+    coef = torch.full((T,), 0.01, device=DEV)
+    flags2 = api.new_flags()
+    grad, tl, loss = api.loss_grad_logits(logits, ids, mask, lse, None, coef, 0.2, V=V, flags=flags2)
+    g = grad[:, :V].float()
+    assert torch.all(g[1] == 0) and torch.all(g[2] == 0) and torch.all(g[5] == 0)
+    assert api.read_flags(flags2) & acrl.FLAG_BAD_ID
+
+
+def test_bad_offsets_flagged():
+    T = 10
+    lp = torch.zeros(T, device=DEV)
+    so = torch.tensor([0, 6, 4, 10], dtype=torch.int64, device=DEV)
+    go = torch.tensor([0, 3], dtype=torch.int32, device=DEV)
+    flags = api.new_flags()
+    api.seq_discrepancy(lp, lp, None, so, go, None, flags=flags)
+    assert api.read_flags(flags) & acrl.FLAG_BAD_OFFSETS
+    flags = api.new_flags()
+    so = torch.tensor([0, 4, 9], dtype=torch.int64, device=DEV)      # does not reach T
+    go = torch.tensor([0, 2], dtype=torch.int32, device=DEV)
+    api.seq_discrepancy(lp, lp, None, so, go, None, flags=flags)
+    assert api.read_flags(flags) & acrl.FLAG_BAD_OFFSETS
+    flags = api.new_flags()
+    so = torch.tensor([0, 4, 10], dtype=torch.int64, device=DEV)
+    go = torch.tensor([0, 3], dtype=torch.int32, device=DEV)         # beyond S
+    api.grpo_advantage(torch.zeros(2, device=DEV), go, acrl.Params(), flags=flags)
+    assert api.read_flags(flags) & acrl.FLAG_BAD_OFFSETS
+
+
+def test_invalid_arguments_rejected_on_host():
+    logits, ids = _tiny_manual(4, 16)
+    with pytest.raises(acrl.AcrlError):
+        api.token_stats(logits[:, 1:], ids, None, V=15)        # misaligned rows
+    with pytest.raises(acrl.AcrlError):
+        api.grpo_advantage(torch.zeros(2, device=DEV), torch.tensor([0, 2], dtype=torch.int32, device=DEV),
+                           acrl.Params(C=1.0))
+
+
+# --------------------------------------------------------------------------
+# controller trajectory: 50 steps with fresh batches (long-response shapes)
+# --------------------------------------------------------------------------
+
+def test_controller_trajectory_50_steps():
+    spec = W.small_variant(W.LONG, name="traj", len_lo=512, len_hi=2048, perturb_frac=0.1, perturb_std=0.3)
+    p = acrl.Params()
+    op = oracle_params(p)
+    state = api.controller_init(p)
+    ost = O.controller_init(op)
+    Xs = []
+    for k in range(50):
+        d = W.token_level(spec, W.seed_for("long", k), device=DEV)
+        disc = api.seq_discrepancy(d["logp_pi"], d["logp_mu"], d["mask"], d["seq_offsets"], d["group_offsets"])
+        adv = api.grpo_advantage(d["rewards"], d["group_offsets"], p)
+        w, coef, alpha = api.controller_step(state, p, disc, d["mask"], d["seq_offsets"], d["group_offsets"], adv)
+        torch.cuda.synchronize()
+        lr, dd, seq, grp, batch, _ = O.seq_discrepancy(host(d["logp_pi"]).astype(np.float64),
+                                                       host(d["logp_mu"]).astype(np.float64), host(d["mask"]),
+                                                       host(d["seq_offsets"]), host(d["group_offsets"]))
+        oadv = O.grpo_advantage(host(d["rewards"]).astype(np.float64), host(d["group_offsets"]), op)
+        ow, oalpha, ost, info, _ = O.controller_step(ost, op, lr, host(d["mask"]), host(d["seq_offsets"]),
+                                                     host(d["group_offsets"]), seq, grp, batch, oadv)
+        st = api.read_state(state)
+        assert int(st["step"]) == k + 1 and int(st["calibrated"]) == 1
+        assert_close_rel(st["X"], ost.X, floor=1e-12, what=f"X step {k}")
+        assert_close_rel(host(w), ow, floor=1e-7, what=f"weight step {k}")
+        assert_close_rel(host(alpha), oalpha, floor=1e-6, what=f"alpha step {k}")
+        Xs.append(float(st["X"]))
+    assert all(x == Xs[0] for x in Xs)     # frozen after step 0, bit for bit
