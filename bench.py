@@ -317,7 +317,7 @@ def run_ours(args):
 
     e2e = None
     if not args.no_e2e and rank == 0:
-        e2e = run_e2e(batch, params, args, dev)
+        e2e = run_e2e(batch, step, params, args, dev)
     if world > 1:
         dist.barrier()
     if rank != 0:
@@ -351,60 +351,131 @@ def run_ours(args):
     return 0
 
 
-def run_e2e(batch, params, args, dev):
-    """Same metric through the public API with host buffers: every step copies
-    the step's inputs from pinned host memory, runs the path and copies the
-    gradient and the loss back."""
+def run_e2e(batch, step, params, args, dev):
+    """Same metric through the public API with the user's buffers in host
+    memory: every step uploads that step's inputs from page-locked host memory,
+    runs the whole path and downloads the gradient and the loss.  Rows move in
+    chunks on two copy streams so that uploads overlap the statistics kernel,
+    downloads overlap the gradient kernel, and one step's downloads overlap the
+    next step's uploads; events order every reuse of a device or host chunk."""
     import torch
 
     import paper_2607_24062_gb300 as acrl
+    cudart = torch.cuda.cudart()
     T, ld = batch.logits.shape
-    host = {
-        "logits": torch.empty((T, ld), dtype=torch.bfloat16, pin_memory=True),
-        "ids": batch.ids.cpu().pin_memory(), "mask": batch.mask.cpu().pin_memory(),
-        "logp_mu": batch.logp_mu.cpu().pin_memory(), "rewards": batch.rewards.cpu().pin_memory(),
-        "seq_offsets": batch.seq_offsets.cpu().pin_memory(), "group_offsets": batch.group_offsets.cpu().pin_memory(),
-    }
-    host["logits"].copy_(batch.logits)
-    grad_host = torch.empty((T, ld), dtype=torch.bfloat16, pin_memory=True)
-    loss_host = torch.empty(1, dtype=torch.float32, pin_memory=True)
-    devbuf = {k: torch.empty_like(v, device=dev) for k, v in host.items() if k != "logits"}
-    devbuf["logits"] = batch.logits  # reuse the resident buffer as the upload target
-    step = acrl.AcrlStep.for_batch(batch, params, device=dev)
-    stream = torch.cuda.current_stream(dev)
+    V = batch.V
+    # the user's host arrays, page-locked in place (torch's pinned allocator would round 44.8 GB up to 64 GB)
+    h_logits_np = np.empty((T, ld), dtype=np.uint16)
+    h_grad_np = np.empty((T, ld), dtype=np.uint16)
+    registered = []
+    try:
+        for arr in (h_logits_np, h_grad_np):
+            rc = cudart.cudaHostRegister(arr.ctypes.data, arr.nbytes, 0)
+            if int(rc) != 0:
+                return {"value": None, "unit": UNIT, "error": f"cudaHostRegister failed ({int(rc)})"}
+            registered.append(arr)
+        h_logits = torch.from_numpy(h_logits_np).view(torch.bfloat16)
+        h_grad = torch.from_numpy(h_grad_np).view(torch.bfloat16)
+        h_logits.copy_(batch.logits)
+        small_h = {k: getattr(batch, k).cpu().pin_memory()
+                   for k in ("ids", "mask", "logp_mu", "rewards", "seq_offsets", "group_offsets")}
+        # two device copies of the O(T) inputs, alternating by step parity
+        small_d = [{k: torch.empty_like(v, device=dev) for k, v in small_h.items()} for _ in range(2)]
+        loss_h = torch.empty(1, dtype=torch.float32, pin_memory=True)
+        d_logits = batch.logits
+        comp = torch.cuda.current_stream(dev)
+        s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        nchunk = max(1, args.e2e_chunks)
+        bounds = [(T * k // nchunk, T * (k + 1) // nchunk) for k in range(nchunk)]
+        E = torch.cuda.Event
+        ev_up = [E() for _ in bounds]      # chunk uploaded
+        ev_used = [E() for _ in bounds]    # gradient kernel done reading the chunk's logits
+        ev_grad = [E() for _ in bounds]    # gradient chunk written
+        ev_down = [E() for _ in bounds]    # gradient chunk downloaded
+        ev_small = [E(), E()]
+        ev_done = [E(), E()]               # all of a step's kernels done (by parity)
+        ev_loss = E()
+        count = [0]
 
-    def one():
-        for k, v in host.items():
-            devbuf[k].copy_(v, non_blocking=True)
-        step.run(devbuf["logits"], devbuf["ids"], devbuf["mask"], devbuf["logp_mu"], devbuf["rewards"],
-                 devbuf["seq_offsets"], devbuf["group_offsets"])
-        grad_host.copy_(step.grad, non_blocking=True)
-        loss_host.copy_(step.loss, non_blocking=True)
+        def one():
+            k = count[0]
+            par = k & 1
+            sd = small_d[par]
+            with torch.cuda.stream(s_in):
+                if k >= 2:
+                    s_in.wait_event(ev_done[par])
+                for name, v in small_h.items():
+                    sd[name].copy_(v, non_blocking=True)
+                ev_small[par].record(s_in)
+                for c, (r0, r1) in enumerate(bounds):
+                    if k >= 1:
+                        s_in.wait_event(ev_used[c])
+                    d_logits[r0:r1].copy_(h_logits[r0:r1], non_blocking=True)
+                    ev_up[c].record(s_in)
+            comp.wait_event(ev_small[par])
+            for c, (r0, r1) in enumerate(bounds):
+                comp.wait_event(ev_up[c])
+                acrl.token_stats(d_logits[r0:r1], sd["ids"][r0:r1], sd["mask"][r0:r1], V=V, lse=step.lse[r0:r1],
+                                 logp=step.logp[r0:r1], entropy=step.entropy[r0:r1], flags=step.flags)
+            acrl.seq_discrepancy(step.logp, sd["logp_mu"], sd["mask"], sd["seq_offsets"], sd["group_offsets"],
+                                 step.entropy, out=step.disc, flags=step.flags)
+            acrl.grpo_advantage(sd["rewards"], sd["group_offsets"], params, adv=step.adv, flags=step.flags)
+            acrl.controller_step(step.state, params, step.disc, sd["mask"], sd["seq_offsets"], sd["group_offsets"],
+                                 step.adv, weight=step.weight, coef=step.coef, alpha=step.alpha, flags=step.flags)
+            for c, (r0, r1) in enumerate(bounds):
+                if k >= 1:
+                    comp.wait_event(ev_down[c])
+                acrl.loss_grad_logits(d_logits[r0:r1], sd["ids"][r0:r1], sd["mask"][r0:r1], step.lse[r0:r1], None,
+                                      step.coef[r0:r1], params.clip_eps, V=V, grad=step.grad[r0:r1],
+                                      token_loss=step.token_loss[r0:r1], loss=step.chunk_loss, flags=step.flags)
+                ev_used[c].record(comp)
+                ev_grad[c].record(comp)
+                with torch.cuda.stream(s_out):
+                    s_out.wait_event(ev_grad[c])
+                    h_grad[r0:r1].copy_(step.grad[r0:r1], non_blocking=True)
+                    ev_down[c].record(s_out)
+            acrl.reduce_loss(step.token_loss, loss=step.loss)
+            ev_loss.record(comp)
+            ev_done[par].record(comp)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_loss)
+                loss_h.copy_(step.loss, non_blocking=True)
+            count[0] += 1
 
-    one()
-    torch.cuda.synchronize()
-    n = max(1, args.e2e_steps)
-    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    s.record(stream)
-    for _ in range(n):
         one()
-    e.record(stream)
-    torch.cuda.synchronize()
-    ms = s.elapsed_time(e) / n
-    h2d = sum(v.numel() * v.element_size() for v in host.values())
-    d2h = grad_host.numel() * grad_host.element_size() + 4
-    return {"value": int(batch.mask.sum()) / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n}
+        torch.cuda.synchronize()
+        n = max(1, args.e2e_steps)
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(comp)
+        for _ in range(n):
+            one()
+        comp.wait_stream(s_out)   # the last step's gradient and loss are on the host
+        t1.record(comp)
+        torch.cuda.synchronize()
+        ms = t0.elapsed_time(t1) / n
+        ok = bool(torch.equal(h_grad[:, :V].view(torch.int16)[:: max(1, T // 64)].to(dev),
+                              step.grad[:, :V].view(torch.int16)[:: max(1, T // 64)]))
+        h2d = T * ld * 2 + sum(v.numel() * v.element_size() for v in small_h.values())
+        d2h = T * ld * 2 + 4
+        return {"value": int(batch.mask.sum()) / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n, "chunks": nchunk,
+                "host_link_GB/s": (h2d + d2h) / (ms / 1e3) / 1e9, "download_matches_device": ok,
+                "host_memory": "user buffers page-locked with cudaHostRegister"}
+    finally:
+        torch.cuda.synchronize()
+        for arr in registered:
+            cudart.cudaHostUnregister(arr.ctypes.data)
 
 
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="qwen")
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=4)
+    ap.add_argument("--e2e-chunks", type=int, default=16)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--ref-seconds", type=float, default=10.0)

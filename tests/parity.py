@@ -111,3 +111,10 @@ def compare_batch(gb, rb, what="batch"):
         assert_close_rel(gb[k], rb[k], floor=1e-9, what=f"{what}.{k}")
     assert_close_rel(gb["H_mean"], rb["H_mean"], floor=1e-5, what=f"{what}.H_mean")
     assert_close_abs(gb["lr_mean"], rb["lr_mean"], TOL_LOGP, what=f"{what}.lr_mean")
+
+
+def assert_loss(got, ref, ref_token_loss, what="loss"):
+    """Scalar loss: 1e-3 relative, with a floor of 1e-6 * sum |token loss| for
+    batches whose token losses cancel (e.g. every weight 1: sum_i A_i = 0)."""
+    floor = 1e-6 * float(np.nansum(np.abs(np.asarray(ref_token_loss, dtype=np.float64)))) + 1e-30
+    assert_close_rel(got, ref, floor=floor, what=what)

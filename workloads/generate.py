@@ -71,7 +71,11 @@ QWEN = WorkloadSpec("qwen", 16, 8, 256, 2048, 151936, dist="student_t", scale=2.
 LONG = WorkloadSpec("long", 8, 4, 4096, 16384, 151936, dist="normal", scale=2.0,
                     fp8_scale="tensor", reward_p=0.3, chunk_rows=65536)
 
-SPECS = {s.name: s for s in (TINY, GRPO, QWEN, LONG)}
+# The Qwen workload at 8,192 rows (2.5 GB of logits): small enough for a full
+# profiler capture, still far larger than L2.
+QWEN_PROFILE = replace(QWEN, name="qwen_profile", n_prompts=2, group_size=4, len_lo=1024, len_hi=1024)
+
+SPECS = {s.name: s for s in (TINY, GRPO, QWEN, LONG, QWEN_PROFILE)}
 BASE_SEED = 2607_24062
 
 
