@@ -40,7 +40,7 @@
 extern "C" {
 #endif
 
-#define ACRL_ABI_VERSION 1
+#define ACRL_ABI_VERSION 2
 
 typedef uint16_t acrl_bf16;                 /* IEEE bfloat16 bit pattern */
 typedef struct CUstream_st* acrl_stream;    /* identical to cudaStream_t */
@@ -64,7 +64,11 @@ typedef enum {
     ACRL_MODE_NONE = 0,   /* plain GRPO (Eq. grpo_objective): w = 1             */
     ACRL_MODE_TIS = 1,    /* token-level truncated IS (Eq. TIS): min(pi/mu, C)  */
     ACRL_MODE_MIS = 2,    /* sequence-level masked IS (Eq. MIS): rho_i 1{rho_i<=C} */
-    ACRL_MODE_ACRL = 3    /* Eq. ACRL: min((pi/mu)^alpha, C)                    */
+    ACRL_MODE_ACRL = 3,   /* Eq. ACRL: min((pi/mu)^alpha, C)                    */
+    ACRL_MODE_ACRL_CONTINUOUS = 4, /* Sec. 5.5 ablation "continuous reduction":
+                                      alpha = -kappa sign(A), no Y/X comparison   */
+    ACRL_MODE_ACRL_FALLBACK = 5    /* Sec. 5.5 ablation "fallback to GRPO": the ACRL
+                                      alpha when Y > X, alpha = 0 (w = 1) otherwise */
 } acrl_mode;
 
 /* Which discrepancy plays Y in alpha = gamma sign(A) (1 - Y/X) (Sec. 4.1). */
@@ -84,12 +88,19 @@ typedef enum {
     ACRL_SINGLETON_ZERO = 1           /* a prompt with one response: A = 0 */
 } acrl_singleton_rule;
 
-/* Hyper-parameters (host memory, read at call time).  48 bytes. */
+/* Hyper-parameters (host memory, read at call time).  64 bytes. */
 typedef struct acrl_params {
     float   gamma;          /* control strength gamma > 0 (Sec. 4.1; 0.35 / 0.65 in Sec. 5.1) */
     float   C;              /* truncation cap C > 1 (Sec. 4.1; 3, or 5 in Sec. 5.3)           */
     float   clip_eps;       /* clip range eps in [0, 1) of Eq. grpo_objective                 */
     float   adv_eps;        /* added to the GRPO std, >= 0                                    */
+    float   kappa;          /* |alpha| > 0 of ACRL_MODE_ACRL_CONTINUOUS (1 or 3 in Sec. 5.5)  */
+    float   x_ema;          /* 0: X frozen once calibrated (the paper's method).  In (0, 1]:
+                               after every later step X <- (1 - x_ema) X + x_ema Y_mean, the
+                               moving-average X the Limitations section suggests           */
+    float   entropy_coeff;  /* beta >= 0: entropy bonus -beta H_t / norm_t added to the loss
+                               (the actor entropy_coeff of App. A; not part of Eq. ACRL)   */
+    float   reserved;       /* must be 0 */
     int32_t mode;           /* acrl_mode                                                      */
     int32_t y_gran;         /* acrl_y_granularity                                             */
     int32_t agg;            /* acrl_agg                                                       */
@@ -252,6 +263,13 @@ acrl_status acrl_controller_init(acrl_controller_state* state, const acrl_params
  *   weight    device float [T] output w_t (0 where m_t = 0).
  *   coef      device float [T] output coef_t (0 where m_t = 0).
  *   alpha     device float [S] output, or NULL.
+ *   ent_coef  device float [T] output beta m_t / norm_t for the entropy bonus,
+ *             or NULL (then p->entropy_coeff is not used).
+ * Ablations (Sec. 5.5): ACRL_MODE_ACRL_CONTINUOUS uses alpha = -kappa sign(A_i);
+ * ACRL_MODE_ACRL_FALLBACK uses the ACRL alpha when Y > X and 0 otherwise.
+ * With p->x_ema > 0, every step after the one that fixed X (or every step, if
+ * X_init > 0) ends with X <- (1 - x_ema) X + x_ema Y_mean; batch->X reports
+ * the X this step used.
  */
 acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params* p,
                                  const float* lr, const uint8_t* mask, int64_t T,
@@ -259,7 +277,7 @@ acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params
                                  const int32_t* group_offsets, int32_t Gn,
                                  acrl_seq_stats* seq, const acrl_group_stats* grp,
                                  acrl_batch_stats* batch, const float* adv,
-                                 float* weight, float* coef, float* alpha,
+                                 float* weight, float* coef, float* alpha, float* ent_coef,
                                  int32_t* dev_flags, acrl_stream stream);
 
 /*
@@ -270,8 +288,12 @@ acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params
  *     grad[t, j]   = coef_t g_t r_t (p_tj - 1[j = a_t])          (bf16)
  *     token_loss_t = -coef_t * (coef_t >= 0 ? min(r, clip(r)) : max(r, clip(r)))
  *     *loss        = sum_t token_loss_t   (fixed order, fp64 accumulation)
- * The probabilities are never stored.  Rows with m_t = 0, coef_t = 0 or
- * g_t = 0 get a zero gradient row without reading their logits.
+ * With an entropy bonus (ent_coef and entropy given, e_t = ent_coef_t):
+ *     grad[t, j]  += e_t p_tj (log p_tj + H_t),   token_loss_t += -e_t H_t
+ * (H_t = -sum_j p_tj log p_tj; d H / d z_j = -p_j (log p_j + H)).
+ * The probabilities are never stored.  Rows with m_t = 0, or with no
+ * gradient (coef_t g_t = 0 and no entropy bonus), get a zero gradient row
+ * without reading the rest of their logits.
  *   logits  device bf16 [T, ld];  grad  device bf16 [T, ld] output (columns
  *           >= V untouched).  May be called on a chunk of rows: every
  *           per-token pointer then points at the chunk's first row.
@@ -281,12 +303,15 @@ acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params
  *           over each row).
  *   old_logp  device float [T] log pi_old(a_t), or NULL for r = 1.
  *   coef    device float [T] from acrl_controller_step.
+ *   entropy, ent_coef  device float [T] (acrl_token_stats' entropy and
+ *           acrl_controller_step's ent_coef), both NULL for no entropy bonus.
  *   clip_eps  the eps of Eq. grpo_objective.
  *   token_loss  device float [T] output;  loss  device float [1] output.
  */
 acrl_status acrl_loss_grad_logits(const acrl_bf16* logits, int64_t T, int64_t V, int64_t ld,
                                   const int32_t* ids, const uint8_t* mask, const float* lse,
-                                  const float* old_logp, const float* coef, float clip_eps,
+                                  const float* old_logp, const float* coef,
+                                  const float* entropy, const float* ent_coef, float clip_eps,
                                   acrl_bf16* grad, float* token_loss, float* loss,
                                   int32_t* dev_flags, acrl_stream stream);
 

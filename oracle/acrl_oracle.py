@@ -48,8 +48,10 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
-# Weight modes (Sec. 2.2 TIS / MIS, Sec. 4.1 ACRL, plain GRPO).
+# Weight modes (Sec. 2.2 TIS / MIS, Sec. 4.1 ACRL, plain GRPO) and the two
+# one-sided ablations of Sec. 5.5.
 MODE_NONE, MODE_TIS, MODE_MIS, MODE_ACRL = 0, 1, 2, 3
+MODE_ACRL_CONTINUOUS, MODE_ACRL_FALLBACK = 4, 5
 # Granularity of the current discrepancy Y.
 Y_GROUP, Y_SEQUENCE, Y_BATCH = 0, 1, 2
 # Loss aggregation.
@@ -73,6 +75,9 @@ class Params:
     C: float = 3.0
     clip_eps: float = 0.2
     adv_eps: float = 1e-6
+    kappa: float = 1.0          # |alpha| of the continuous-reduction ablation (Sec. 5.5)
+    x_ema: float = 0.0          # moving-average X (Limitations); 0 keeps X frozen
+    entropy_coeff: float = 0.0  # entropy bonus beta (App. A actor.entropy_coeff)
     mode: int = MODE_ACRL
     y_gran: int = Y_GROUP
     agg: int = AGG_SEQ_MEAN_TOKEN_MEAN
@@ -317,6 +322,7 @@ def controller_step(state: ControllerState, params: Params, lr, mask, seq_offset
     flags = 0
 
     applying = True
+    was_calibrated = st.calibrated
     if not st.calibrated:
         st.calib_sum += batch["Y_sum"]
         st.calib_count += batch["n_groups_valid"]
@@ -329,8 +335,11 @@ def controller_step(state: ControllerState, params: Params, lr, mask, seq_offset
     st.step += 1
 
     X = st.X
-    if params.mode == MODE_ACRL and applying and not X > 0:
+    if params.mode in (MODE_ACRL, MODE_ACRL_FALLBACK) and applying and not X > 0:
         flags |= FLAG_X_NONPOS
+    # Moving-average X (Limitations): this step uses X, later steps the update.
+    if was_calibrated and params.x_ema > 0:
+        st.X = (1.0 - params.x_ema) * X + params.x_ema * batch["Y_mean"]
 
     logC = math.log(params.C)
     alpha = np.zeros(S)
@@ -340,7 +349,10 @@ def controller_step(state: ControllerState, params: Params, lr, mask, seq_offset
         n_i = int(seq["n"][i])
         if params.mode == MODE_TIS or params.mode == MODE_MIS:
             alpha[i] = 1.0
-        elif params.mode == MODE_ACRL and applying and X > 0 and n_i > 0:
+        elif params.mode == MODE_ACRL_CONTINUOUS and n_i > 0:
+            # Sec. 5.5: alpha = -1 (or -3) where A > 0, +1 (or +3) where A < 0
+            alpha[i] = -params.kappa * np.sign(A[i])
+        elif params.mode in (MODE_ACRL, MODE_ACRL_FALLBACK) and applying and X > 0 and n_i > 0:
             if params.y_gran == Y_GROUP:
                 Y = grp["Y"][seq["group"][i]]
             elif params.y_gran == Y_SEQUENCE:
@@ -348,6 +360,8 @@ def controller_step(state: ControllerState, params: Params, lr, mask, seq_offset
             else:
                 Y = batch["Y_mean"]
             alpha[i] = params.gamma * np.sign(A[i]) * (1.0 - Y / X)
+            if params.mode == MODE_ACRL_FALLBACK and not Y > X:
+                alpha[i] = 0.0      # Sec. 5.5: plain GRPO update when Y < X
         for t in range(so[i], so[i + 1]):
             if not m[t]:
                 continue
@@ -441,14 +455,23 @@ def loss_grad_logits(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq,
         rc = min(max(r, 1.0 - eps), 1.0 + eps)
         surrogate = min(r * Ai, rc * Ai)
         token_loss[t] = -w[t] * surrogate / norm
-        total.append(token_loss[t])
         gate = (Ai >= 0 and r <= 1.0 + eps) or (Ai < 0 and r >= 1.0 - eps)
         coef = w[t] * (1.0 if gate else 0.0) * r * Ai / norm
-        if coef == 0.0:
+        beta = params.entropy_coeff / norm
+        if coef == 0.0 and beta == 0.0:
+            total.append(token_loss[t])
             continue
-        p = np.exp(row - lse_t)
-        p[a] -= 1.0
-        grad[k] = coef * p
+        logq = row - lse_t
+        p = np.exp(logq)
+        g = coef * p
+        g[a] -= coef
+        if beta != 0.0:
+            # entropy bonus -beta H_t / norm_t; dH/dz_j = -p_j (log p_j + H)
+            H_t = -np.sum(p * logq)
+            token_loss[t] -= beta * H_t
+            g += beta * p * (logq + H_t)
+        total.append(token_loss[t])
+        grad[k] = g
     return grad, token_loss, math.fsum(total)
 
 
@@ -486,9 +509,22 @@ def loss_coefficients(weight, adv, mask, seq_offsets, seq, grp, batch, params: P
     return coef
 
 
-def surrogate_loss(logp, old_logp, adv, weight, mask, seq_offsets, seq, grp, batch, params: Params):
+def entropy_coefficients(mask, seq_offsets, seq, grp, batch, params: Params):
+    """Per-token factor beta / norm_t of the entropy bonus (0 on masked tokens)."""
+    so = np.asarray(seq_offsets, dtype=np.int64)
+    T = int(so[-1])
+    m = np.ones(T, dtype=bool) if mask is None else (np.asarray(mask) != 0)
+    owner, norm = _norms(mask, seq_offsets, seq, grp, batch, params)
+    out = np.zeros(T)
+    ok = m & (owner >= 0) & (norm > 0)
+    out[ok] = params.entropy_coeff / norm[ok]
+    return out
+
+
+def surrogate_loss(logp, old_logp, adv, weight, mask, seq_offsets, seq, grp, batch, params: Params, entropy=None):
     """Token losses -w_t min(r A, clip(r) A) / norm_t of Eq. ACRL from the
-    current log-probs alone (r = exp(logp - old_logp), or 1 without old_logp).
+    current log-probs alone (r = exp(logp - old_logp), or 1 without old_logp),
+    minus beta H_t / norm_t when an entropy bonus and the entropies are given.
     Returns (token_loss [T], total)."""
     w = np.asarray(weight, dtype=np.float64)
     A = np.asarray(adv, dtype=np.float64)
@@ -504,6 +540,8 @@ def surrogate_loss(logp, old_logp, adv, weight, mask, seq_offsets, seq, grp, bat
         r = 1.0 if old_logp is None else math.exp(float(logp[t]) - float(old_logp[t]))
         rc = min(max(r, 1.0 - eps), 1.0 + eps)
         tl[t] = -w[t] * min(r * A[i], rc * A[i]) / norm[t]
+        if entropy is not None and params.entropy_coeff:
+            tl[t] -= params.entropy_coeff * float(entropy[t]) / norm[t]
     return tl, math.fsum(tl)
 
 

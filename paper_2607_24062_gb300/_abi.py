@@ -21,7 +21,7 @@ c_i32, c_i64, c_f32, c_f64, c_p = ctypes.c_int32, ctypes.c_int64, ctypes.c_float
 # status codes, flag bits and enums (values fixed by include/acrl.h)
 OK, ERR_INVALID_ARG, ERR_CUDA, ERR_NOT_IMPLEMENTED, ERR_DEVICE_FLAGS = 0, 1, 2, 3, 4
 FLAG_BAD_ID, FLAG_NONFINITE, FLAG_BAD_OFFSETS, FLAG_X_NONPOS = 0x1, 0x2, 0x4, 0x8
-MODE_NONE, MODE_TIS, MODE_MIS, MODE_ACRL = 0, 1, 2, 3
+MODE_NONE, MODE_TIS, MODE_MIS, MODE_ACRL, MODE_ACRL_CONTINUOUS, MODE_ACRL_FALLBACK = 0, 1, 2, 3, 4, 5
 Y_GROUP, Y_SEQUENCE, Y_BATCH = 0, 1, 2
 AGG_SEQ_MEAN_TOKEN_MEAN, AGG_TOKEN_MEAN = 0, 1
 SINGLETON_MEAN0_STD1, SINGLETON_ZERO = 0, 1
@@ -30,15 +30,16 @@ SINGLETON_MEAN0_STD1, SINGLETON_ZERO = 0, 1
 class Params(ctypes.Structure):
     """acrl_params.  Defaults: gamma 0.65 and C 3 as in Sec. 5.1 of the paper."""
 
-    _fields_ = [("gamma", c_f32), ("C", c_f32), ("clip_eps", c_f32), ("adv_eps", c_f32), ("mode", c_i32),
+    _fields_ = [("gamma", c_f32), ("C", c_f32), ("clip_eps", c_f32), ("adv_eps", c_f32), ("kappa", c_f32),
+                ("x_ema", c_f32), ("entropy_coeff", c_f32), ("reserved", c_f32), ("mode", c_i32),
                 ("y_gran", c_i32), ("agg", c_i32), ("adv_ddof", c_i32), ("singleton_rule", c_i32),
                 ("calib_steps", c_i32), ("X_init", c_f64)]
 
-    def __init__(self, gamma=0.65, C=3.0, clip_eps=0.2, adv_eps=1e-6, mode=MODE_ACRL, y_gran=Y_GROUP,
-                 agg=AGG_SEQ_MEAN_TOKEN_MEAN, adv_ddof=1, singleton_rule=SINGLETON_MEAN0_STD1, calib_steps=1,
-                 X_init=0.0):
-        super().__init__(gamma, C, clip_eps, adv_eps, mode, y_gran, agg, adv_ddof, singleton_rule, calib_steps,
-                         X_init)
+    def __init__(self, gamma=0.65, C=3.0, clip_eps=0.2, adv_eps=1e-6, kappa=1.0, x_ema=0.0, entropy_coeff=0.0,
+                 mode=MODE_ACRL, y_gran=Y_GROUP, agg=AGG_SEQ_MEAN_TOKEN_MEAN, adv_ddof=1,
+                 singleton_rule=SINGLETON_MEAN0_STD1, calib_steps=1, X_init=0.0):
+        super().__init__(gamma, C, clip_eps, adv_eps, kappa, x_ema, entropy_coeff, 0.0, mode, y_gran, agg, adv_ddof,
+                         singleton_rule, calib_steps, X_init)
 
     def as_dict(self):
         return {k: getattr(self, k) for k, _ in self._fields_}
@@ -66,9 +67,9 @@ SIGNATURES = {
     "acrl_grpo_advantage": (c_i32, [c_p, c_p, c_i32, c_i32, ctypes.POINTER(Params), c_p, c_p, c_p]),
     "acrl_controller_init": (c_i32, [c_p, ctypes.POINTER(Params), c_p]),
     "acrl_controller_step": (c_i32, [c_p, ctypes.POINTER(Params), c_p, c_p, c_i64, c_p, c_i32, c_p, c_i32, c_p, c_p,
-                                     c_p, c_p, c_p, c_p, c_p, c_p, c_p]),
-    "acrl_loss_grad_logits": (c_i32, [c_p, c_i64, c_i64, c_i64, c_p, c_p, c_p, c_p, c_p, c_f32, c_p, c_p, c_p, c_p,
-                                      c_p]),
+                                     c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p]),
+    "acrl_loss_grad_logits": (c_i32, [c_p, c_i64, c_i64, c_i64, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_f32, c_p, c_p,
+                                      c_p, c_p, c_p]),
     "acrl_reduce_loss": (c_i32, [c_p, c_i64, c_p, c_p]),
     "acrl_read_flags": (c_i32, [c_p, ctypes.POINTER(c_i32), c_p]),
 }

@@ -153,8 +153,9 @@ def read_state(state: torch.Tensor) -> np.void:
 
 
 def controller_step(state, params: Params, disc: Discrepancy, mask, seq_offsets, group_offsets, adv, *, weight=None,
-                    coef=None, alpha=None, flags=None, stream=None):
-    """acrl_controller_step.  Returns (weight [T], coef [T], alpha [S])."""
+                    coef=None, alpha=None, ent_coef=None, flags=None, stream=None):
+    """acrl_controller_step.  Returns (weight [T], coef [T], alpha [S]); the
+    entropy-bonus factors go to `ent_coef` [T] when given."""
     T = disc.lr.numel()
     dev = disc.lr.device
     weight = torch.empty(T, dtype=torch.float32, device=dev) if weight is None else _need(weight, torch.float32, T, "weight")
@@ -163,17 +164,20 @@ def controller_step(state, params: Params, disc: Discrepancy, mask, seq_offsets,
         _need(alpha, torch.float32, disc.S, "alpha")
     _need(adv, torch.float32, disc.S, "adv")
     _opt(mask, torch.uint8, T, "mask")
+    _opt(ent_coef, torch.float32, T, "ent_coef")
     flags = new_flags(dev) if flags is None else flags
     check(lib().acrl_controller_step(_ptr(state), ctypes.byref(params), _ptr(disc.lr), _ptr(mask), T,
                                      _ptr(seq_offsets), disc.S, _ptr(group_offsets), disc.Gn, _ptr(disc.seq),
                                      _ptr(disc.grp), _ptr(disc.batch), _ptr(adv), _ptr(weight), _ptr(coef),
-                                     _ptr(alpha), _ptr(flags), _stream(stream)), "acrl_controller_step")
+                                     _ptr(alpha), _ptr(ent_coef), _ptr(flags), _stream(stream)),
+          "acrl_controller_step")
     return weight, coef, alpha
 
 
-def loss_grad_logits(logits, ids, mask, lse, old_logp, coef, clip_eps: float, *, V=None, grad=None, token_loss=None,
-                     loss=None, flags=None, stream=None):
-    """acrl_loss_grad_logits.  Returns (grad bf16 [T, ld], token_loss [T], loss [1])."""
+def loss_grad_logits(logits, ids, mask, lse, old_logp, coef, clip_eps: float, *, V=None, entropy=None, ent_coef=None,
+                     grad=None, token_loss=None, loss=None, flags=None, stream=None):
+    """acrl_loss_grad_logits.  Returns (grad bf16 [T, ld], token_loss [T], loss [1]).
+    `entropy` and `ent_coef` (both or neither) add the entropy bonus."""
     T, ld = _rows(logits, "logits")
     V = ld if V is None else V
     dev = logits.device
@@ -182,6 +186,8 @@ def loss_grad_logits(logits, ids, mask, lse, old_logp, coef, clip_eps: float, *,
     _opt(lse, torch.float32, T, "lse")
     _opt(old_logp, torch.float32, T, "old_logp")
     _need(coef, torch.float32, T, "coef")
+    _opt(entropy, torch.float32, T, "entropy")
+    _opt(ent_coef, torch.float32, T, "ent_coef")
     if grad is None:
         grad = torch.empty((T, ld), dtype=torch.bfloat16, device=dev)
     elif grad.dtype != torch.bfloat16 or grad.dim() != 2 or grad.stride(0) != ld or grad.stride(1) != 1 or \
@@ -192,8 +198,9 @@ def loss_grad_logits(logits, ids, mask, lse, old_logp, coef, clip_eps: float, *,
     loss = torch.empty(1, dtype=torch.float32, device=dev) if loss is None else _need(loss, torch.float32, 1, "loss")
     flags = new_flags(dev) if flags is None else flags
     check(lib().acrl_loss_grad_logits(_ptr(logits), T, V, ld, _ptr(ids), _ptr(mask), _ptr(lse), _ptr(old_logp),
-                                      _ptr(coef), float(clip_eps), _ptr(grad), _ptr(token_loss), _ptr(loss),
-                                      _ptr(flags), _stream(stream)), "acrl_loss_grad_logits")
+                                      _ptr(coef), _ptr(entropy), _ptr(ent_coef), float(clip_eps), _ptr(grad),
+                                      _ptr(token_loss), _ptr(loss), _ptr(flags), _stream(stream)),
+          "acrl_loss_grad_logits")
     return grad, token_loss, loss
 
 

@@ -28,8 +28,9 @@ inline acrl_status launch_status() {
 inline bool params_ok(const acrl_params* p) {
     if (!p) return false;
     if (!(p->gamma > 0.f) || !(p->C > 1.f) || !(p->clip_eps >= 0.f && p->clip_eps < 1.f)) return false;
-    if (!(p->adv_eps >= 0.f)) return false;
-    if (p->mode < ACRL_MODE_NONE || p->mode > ACRL_MODE_ACRL) return false;
+    if (!(p->adv_eps >= 0.f) || !(p->kappa > 0.f) || !(p->x_ema >= 0.f && p->x_ema <= 1.f)) return false;
+    if (!(p->entropy_coeff >= 0.f) || p->reserved != 0.f) return false;
+    if (p->mode < ACRL_MODE_NONE || p->mode > ACRL_MODE_ACRL_FALLBACK) return false;
     if (p->y_gran < ACRL_Y_GROUP || p->y_gran > ACRL_Y_BATCH) return false;
     if (p->agg < ACRL_AGG_SEQ_MEAN_TOKEN_MEAN || p->agg > ACRL_AGG_TOKEN_MEAN) return false;
     if (p->adv_ddof < 0 || p->adv_ddof > 1) return false;

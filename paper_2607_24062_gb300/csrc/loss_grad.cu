@@ -8,9 +8,11 @@
 // - log2|c|)), so each element costs one FMA and one SFU exp2; the sign is
 // applied to the packed bf16 pair with one XOR.  The target column is written
 // as c * expm1(logp) so that p_a - 1 keeps its accuracy when p_a is near 1.
-// Rows that carry no gradient (masked, zero coefficient, clipped) are written
-// as zeros without reading their logits.  With lse == NULL the row's
-// log-sum-exp is first recomputed by a sweep over the same row.
+// With an entropy bonus e_t the element becomes p (c + e (z - lse + H)): one
+// more FMA and a multiply.  Rows that carry no gradient (masked, zero
+// coefficient and no bonus, clipped) are written as zeros without reading
+// their logits.  With lse == NULL the row's log-sum-exp is first recomputed
+// by a sweep over the same row.
 #include "acrl_device.cuh"
 #include "acrl_host.h"
 #include "row_lse.cuh"
@@ -20,28 +22,43 @@ namespace {
 
 constexpr uint32_t kSignPair = 0x80008000u;
 
+// Per-row constants of the streaming pass.
 struct RowPlan {
-    float B;        // lse log2e - log2|c|
-    uint32_t sgn;   // kSignPair when c < 0
-    float target;   // gradient at the sampled column, sign included
+    float B;        // policy term only: lse log2e - log2|c|
+    uint32_t sgn;   // policy term only: kSignPair when c < 0
+    float L2;       // with entropy: lse log2e
+    float e;        // with entropy: e_t
+    float c2;       // with entropy: c - e (lse - H)
+    float target;   // gradient at the sampled column
     int a;          // sampled column
 };
 
+template <bool ENT>
+__device__ __forceinline__ float grad_elem(float z, const RowPlan& rp) {
+    if (ENT) {
+        const float p = ex2(fmaf(z, kLog2e, -rp.L2));
+        return p * fmaf(rp.e, z, rp.c2);
+    }
+    return ex2(fmaf(z, kLog2e, -rp.B));  // magnitude; sign applied by the caller
+}
+
+template <bool ENT>
 __device__ __forceinline__ uint4 grad_vec(const uint4 v, const RowPlan& rp, int rel) {
     float e[8];
-    e[0] = ex2(fmaf(bf16_lo(v.x), kLog2e, -rp.B));
-    e[1] = ex2(fmaf(bf16_hi(v.x), kLog2e, -rp.B));
-    e[2] = ex2(fmaf(bf16_lo(v.y), kLog2e, -rp.B));
-    e[3] = ex2(fmaf(bf16_hi(v.y), kLog2e, -rp.B));
-    e[4] = ex2(fmaf(bf16_lo(v.z), kLog2e, -rp.B));
-    e[5] = ex2(fmaf(bf16_hi(v.z), kLog2e, -rp.B));
-    e[6] = ex2(fmaf(bf16_lo(v.w), kLog2e, -rp.B));
-    e[7] = ex2(fmaf(bf16_hi(v.w), kLog2e, -rp.B));
+    e[0] = grad_elem<ENT>(bf16_lo(v.x), rp);
+    e[1] = grad_elem<ENT>(bf16_hi(v.x), rp);
+    e[2] = grad_elem<ENT>(bf16_lo(v.y), rp);
+    e[3] = grad_elem<ENT>(bf16_hi(v.y), rp);
+    e[4] = grad_elem<ENT>(bf16_lo(v.z), rp);
+    e[5] = grad_elem<ENT>(bf16_hi(v.z), rp);
+    e[6] = grad_elem<ENT>(bf16_lo(v.w), rp);
+    e[7] = grad_elem<ENT>(bf16_hi(v.w), rp);
+    const uint32_t sgn = ENT ? 0u : rp.sgn;
     uint4 o;
     if (static_cast<unsigned>(rel) < 8u) {  // the vector holding the sampled column
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-            const float val = rp.sgn ? -e[j] : e[j];
+            const float val = sgn ? -e[j] : e[j];
             e[j] = (j == rel) ? rp.target : val;
         }
         o.x = pack_bf16x2(e[0], e[1]);
@@ -50,14 +67,14 @@ __device__ __forceinline__ uint4 grad_vec(const uint4 v, const RowPlan& rp, int 
         o.w = pack_bf16x2(e[6], e[7]);
         return o;
     }
-    o.x = pack_bf16x2(e[0], e[1]) ^ rp.sgn;
-    o.y = pack_bf16x2(e[2], e[3]) ^ rp.sgn;
-    o.z = pack_bf16x2(e[4], e[5]) ^ rp.sgn;
-    o.w = pack_bf16x2(e[6], e[7]) ^ rp.sgn;
+    o.x = pack_bf16x2(e[0], e[1]) ^ sgn;
+    o.y = pack_bf16x2(e[2], e[3]) ^ sgn;
+    o.z = pack_bf16x2(e[4], e[5]) ^ sgn;
+    o.w = pack_bf16x2(e[6], e[7]) ^ sgn;
     return o;
 }
 
-template <int TEAM, int UNROLL>
+template <int TEAM, int UNROLL, bool ENT>
 __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ row, acrl_bf16* __restrict__ grow, int V,
                                                 int tid, const RowPlan& rp) {
     const int nvec = V >> 3;
@@ -71,13 +88,13 @@ __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ ro
 #pragma unroll
         for (int k = 0; k < UNROLL; ++k) {
             const int vi = v + k * TEAM;
-            st_stream(dst + vi, grad_vec(buf[k], rp, rp.a - (vi << 3)));
+            st_stream(dst + vi, grad_vec<ENT>(buf[k], rp, rp.a - (vi << 3)));
         }
     }
-    for (; v < nvec; v += TEAM) st_stream(dst + v, grad_vec(ld_stream(src + v), rp, rp.a - (v << 3)));
+    for (; v < nvec; v += TEAM) st_stream(dst + v, grad_vec<ENT>(ld_stream(src + v), rp, rp.a - (v << 3)));
     for (int j = (nvec << 3) + tid; j < V; j += TEAM) {
-        float val = ex2(fmaf(bf16_to_float(row[j]), kLog2e, -rp.B));
-        if (rp.sgn) val = -val;
+        float val = grad_elem<ENT>(bf16_to_float(row[j]), rp);
+        if (!ENT && rp.sgn) val = -val;
         if (j == rp.a) val = rp.target;
         grow[j] = static_cast<acrl_bf16>(pack_bf16x2(val, 0.f) & 0xffffu);
     }
@@ -94,8 +111,7 @@ __device__ __forceinline__ void zero_row(acrl_bf16* __restrict__ grow, int V, in
 
 struct RowCoef {
     float c;       // coef_t g_t r_t
-    float loss;    // token loss
-    float lp;      // logp_t
+    float loss;    // token loss (policy term)
 };
 
 // Scalar part of a live row: r, the clip gate, the coefficient and the loss.
@@ -106,129 +122,151 @@ __device__ __forceinline__ RowCoef row_coef(float c0, float lp, const float* old
     const bool gate = c0 >= 0.f ? (r <= 1.f + eps) : (r >= 1.f - eps);
     RowCoef out;
     out.c = gate ? c0 * r : 0.f;
-    out.loss = -c0 * (c0 >= 0.f ? fminf(r, rc) : fmaxf(r, rc));
-    out.lp = lp;
+    out.loss = c0 == 0.f ? 0.f : -c0 * (c0 >= 0.f ? fminf(r, rc) : fmaxf(r, rc));
     return out;
 }
 
-__device__ __forceinline__ RowPlan make_plan(float c, float L, float lp, int a) {
+template <bool ENT>
+__device__ __forceinline__ RowPlan make_plan(float c, float e, float L, float H, float za, float lp, int a) {
     RowPlan rp;
-    rp.B = fmaf(L, kLog2e, -log2f(fabsf(c)));
-    rp.sgn = c < 0.f ? kSignPair : 0u;
-    rp.target = c * expm1f(lp);
     rp.a = a;
+    if (ENT) {
+        rp.L2 = L * kLog2e;
+        rp.e = e;
+        rp.c2 = fmaf(-e, L - H, c);
+        rp.B = 0.f;
+        rp.sgn = 0u;
+        // c (p_a - 1) + e p_a (z_a - lse + H)
+        rp.target = fmaf(e * expf(lp), za - L + H, c * expm1f(lp));
+    } else {
+        rp.B = fmaf(L, kLog2e, -log2f(fabsf(c)));
+        rp.sgn = c < 0.f ? kSignPair : 0u;
+        rp.L2 = rp.e = rp.c2 = 0.f;
+        rp.target = c * expm1f(lp);
+    }
     return rp;
 }
 
-// A whole CTA per row.
-template <int THREADS, int UNROLL, bool RECOMPUTE>
+// One row handled by a team (a whole CTA, or one warp).  `part` is the CTA's
+// shared scratch for the recompute sweep (unused by warp teams).
+template <int TEAM, int UNROLL, bool RECOMPUTE, bool ENT>
+__device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, int64_t t, int V, int64_t ld,
+                                         const int32_t* __restrict__ ids, const uint8_t* __restrict__ mask,
+                                         const float* __restrict__ lse, const float* __restrict__ old_logp,
+                                         const float* __restrict__ coef, const float* __restrict__ entropy,
+                                         const float* __restrict__ ent_coef, float eps, acrl_bf16* __restrict__ grad,
+                                         float* __restrict__ token_loss, int32_t* flags, int tid, LseAcc* part) {
+    const acrl_bf16* row = logits + t * ld;
+    acrl_bf16* grow = grad + t * ld;
+    const bool m = mask ? mask[t] != 0 : true;
+    const float c0 = coef[t];
+    const float e = ENT ? ent_coef[t] : 0.f;
+    const int a = ids[t];
+    const bool bad_id = a < 0 || a >= V;
+    if (m && bad_id && tid == 0) raise_flag(flags, ACRL_FLAG_BAD_ID);
+    const bool live = m && !bad_id && (c0 != 0.f || e != 0.f);
+    float c = 0.f, loss = 0.f, L = 0.f, H = 0.f, za = 0.f, lp = 0.f;
+    if (live) {
+        if (RECOMPUTE) {
+            float mx;
+            LseAcc acc = warp_lse(row_partial<TEAM, UNROLL>(row, V, tid, mx));
+            if (TEAM > 32) {
+                constexpr int NW = TEAM / 32;
+                if ((tid & 31) == 0) part[tid >> 5] = acc;
+                __syncthreads();
+                acc = part[0];
+#pragma unroll
+                for (int w = 1; w < NW; ++w) acc = lse_merge(acc, part[w]);
+                __syncthreads();
+            }
+            L = kLn2 * (acc.U + log2f(acc.s0));
+        } else {
+            L = lse[t];
+        }
+        za = bf16_to_float(row[a]);
+        lp = za - L;
+        const RowCoef rc = row_coef(c0, lp, old_logp, t, eps);
+        c = rc.c;
+        loss = rc.loss;
+        if (ENT) {
+            H = entropy[t];
+            loss -= e * H;
+        }
+    }
+    if (tid == 0) token_loss[t] = loss;
+    if (c == 0.f && e == 0.f) {
+        zero_row<TEAM>(grow, V, tid);
+    } else {
+        stream_grad_row<TEAM, UNROLL, ENT>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a));
+    }
+}
+
+template <int THREADS, int UNROLL, bool RECOMPUTE, bool ENT>
 __global__ void __launch_bounds__(THREADS) loss_grad_cta(
     const acrl_bf16* __restrict__ logits, int64_t T, int V, int64_t ld, const int32_t* __restrict__ ids,
     const uint8_t* __restrict__ mask, const float* __restrict__ lse, const float* __restrict__ old_logp,
-    const float* __restrict__ coef, float eps, acrl_bf16* __restrict__ grad, float* __restrict__ token_loss,
-    int32_t* flags) {
-    constexpr int NW = THREADS / 32;
-    __shared__ LseAcc part[NW];
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    for (int64_t t = blockIdx.x; t < T; t += gridDim.x) {
-        const acrl_bf16* row = logits + t * ld;
-        acrl_bf16* grow = grad + t * ld;
-        const bool m = mask ? mask[t] != 0 : true;
-        const float c0 = coef[t];
-        const int a = ids[t];
-        const bool bad_id = a < 0 || a >= V;
-        if (m && bad_id && threadIdx.x == 0) raise_flag(flags, ACRL_FLAG_BAD_ID);
-        const bool live = m && c0 != 0.f && !bad_id;
-        RowCoef rc{0.f, 0.f, 0.f};
-        float L = 0.f;
-        if (live) {
-            if (RECOMPUTE) {
-                float mx;
-                LseAcc acc = row_partial<THREADS, UNROLL>(row, V, threadIdx.x, mx);
-                acc = warp_lse(acc);
-                if (lane == 0) part[wid] = acc;
-                __syncthreads();
-                LseAcc r = part[0];
-#pragma unroll
-                for (int w = 1; w < NW; ++w) r = lse_merge(r, part[w]);
-                __syncthreads();
-                L = kLn2 * (r.U + log2f(r.s0));
-            } else {
-                L = lse[t];
-            }
-            rc = row_coef(c0, bf16_to_float(row[a]) - L, old_logp, t, eps);
-        }
-        if (threadIdx.x == 0) token_loss[t] = rc.loss;
-        if (rc.c == 0.f) {
-            zero_row<THREADS>(grow, V, threadIdx.x);
-        } else {
-            stream_grad_row<THREADS, UNROLL>(row, grow, V, threadIdx.x, make_plan(rc.c, L, rc.lp, a));
-        }
-    }
+    const float* __restrict__ coef, const float* __restrict__ entropy, const float* __restrict__ ent_coef, float eps,
+    acrl_bf16* __restrict__ grad, float* __restrict__ token_loss, int32_t* flags) {
+    __shared__ LseAcc part[THREADS / 32];
+    for (int64_t t = blockIdx.x; t < T; t += gridDim.x)
+        grad_row<THREADS, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
+                                                  eps, grad, token_loss, flags, threadIdx.x, part);
 }
 
-// One warp per row.
-template <int THREADS, int UNROLL, bool RECOMPUTE>
+template <int THREADS, int UNROLL, bool RECOMPUTE, bool ENT>
 __global__ void __launch_bounds__(THREADS) loss_grad_warp(
     const acrl_bf16* __restrict__ logits, int64_t T, int V, int64_t ld, const int32_t* __restrict__ ids,
     const uint8_t* __restrict__ mask, const float* __restrict__ lse, const float* __restrict__ old_logp,
-    const float* __restrict__ coef, float eps, acrl_bf16* __restrict__ grad, float* __restrict__ token_loss,
-    int32_t* flags) {
+    const float* __restrict__ coef, const float* __restrict__ entropy, const float* __restrict__ ent_coef, float eps,
+    acrl_bf16* __restrict__ grad, float* __restrict__ token_loss, int32_t* flags) {
     constexpr int NW = THREADS / 32;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    for (int64_t t = int64_t(blockIdx.x) * NW + wid; t < T; t += int64_t(gridDim.x) * NW) {
-        const acrl_bf16* row = logits + t * ld;
-        acrl_bf16* grow = grad + t * ld;
-        const bool m = mask ? mask[t] != 0 : true;
-        const float c0 = coef[t];
-        const int a = ids[t];
-        const bool bad_id = a < 0 || a >= V;
-        if (m && bad_id && lane == 0) raise_flag(flags, ACRL_FLAG_BAD_ID);
-        const bool live = m && c0 != 0.f && !bad_id;
-        RowCoef rc{0.f, 0.f, 0.f};
-        float L = 0.f;
-        if (live) {
-            if (RECOMPUTE) {
-                float mx;
-                LseAcc acc = warp_lse(row_partial<32, UNROLL>(row, V, lane, mx));
-                L = kLn2 * (acc.U + log2f(acc.s0));
-            } else {
-                L = lse[t];
-            }
-            rc = row_coef(c0, bf16_to_float(row[a]) - L, old_logp, t, eps);
-        }
-        if (lane == 0) token_loss[t] = rc.loss;
-        if (rc.c == 0.f) {
-            zero_row<32>(grow, V, lane);
-        } else {
-            stream_grad_row<32, UNROLL>(row, grow, V, lane, make_plan(rc.c, L, rc.lp, a));
-        }
-    }
+    for (int64_t t = int64_t(blockIdx.x) * NW + wid; t < T; t += int64_t(gridDim.x) * NW)
+        grad_row<32, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps,
+                                             grad, token_loss, flags, lane, nullptr);
 }
 
-// Scalar loss: sum of token losses in a fixed order with fp64 accumulation.
+// Scalar loss: sum of token losses in a fixed order.  Each thread adds float4
+// groups (four values in fp32) into two alternating fp64 accumulators, so the
+// loads pipeline and the fp64 adds are a quarter of the values; then a fixed
+// CTA tree in fp64.
 constexpr int kSumThreads = 1024;
 __global__ void __launch_bounds__(kSumThreads) loss_sum_kernel(const float* __restrict__ tl, int64_t T,
                                                                float* __restrict__ loss) {
     __shared__ double sh[kSumThreads / 32];
-    double s = 0.0;
-    for (int64_t t = threadIdx.x; t < T; t += kSumThreads) s += tl[t];
-    s = block_sum<double, kSumThreads / 32>(s, sh);
+    double s0 = 0.0, s1 = 0.0;
+    const bool vec = (reinterpret_cast<uintptr_t>(tl) & 15u) == 0;
+    const int64_t n4 = vec ? T / 4 : 0;
+    const float4* v = reinterpret_cast<const float4*>(tl);
+    int64_t i = threadIdx.x;
+#pragma unroll 4
+    for (; i + kSumThreads < n4; i += 2 * kSumThreads) {
+        const float4 a = v[i], b = v[i + kSumThreads];
+        s0 += double((a.x + a.y) + (a.z + a.w));
+        s1 += double((b.x + b.y) + (b.z + b.w));
+    }
+    for (; i < n4; i += kSumThreads) {
+        const float4 a = v[i];
+        s0 += double((a.x + a.y) + (a.z + a.w));
+    }
+    for (int64_t j = 4 * n4 + threadIdx.x; j < T; j += kSumThreads) s1 += tl[j];
+    double s = block_sum<double, kSumThreads / 32>(s0 + s1, sh);
     if (threadIdx.x == 0) *loss = float(s);
 }
 
-template <bool RECOMPUTE>
+template <bool RECOMPUTE, bool ENT>
 void launch_loss_grad(const acrl_bf16* logits, int64_t T, int V, int64_t ld, const int32_t* ids, const uint8_t* mask,
-                      const float* lse, const float* old_logp, const float* coef, float eps, acrl_bf16* grad,
-                      float* token_loss, int32_t* flags, cudaStream_t s) {
+                      const float* lse, const float* old_logp, const float* coef, const float* entropy,
+                      const float* ent_coef, float eps, acrl_bf16* grad, float* token_loss, int32_t* flags,
+                      cudaStream_t s) {
     if (V <= kWarpRowMaxV) {
         constexpr int THREADS = 256;
-        loss_grad_warp<THREADS, 4, RECOMPUTE><<<unsigned(grid_for(THREADS / 32, T)), THREADS, 0, s>>>(
-            logits, T, V, ld, ids, mask, lse, old_logp, coef, eps, grad, token_loss, flags);
+        loss_grad_warp<THREADS, 4, RECOMPUTE, ENT><<<unsigned(grid_for(THREADS / 32, T)), THREADS, 0, s>>>(
+            logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
     } else {
         constexpr int THREADS = 512;
-        loss_grad_cta<THREADS, 4, RECOMPUTE><<<unsigned(grid_for(1, T)), THREADS, 0, s>>>(
-            logits, T, V, ld, ids, mask, lse, old_logp, coef, eps, grad, token_loss, flags);
+        loss_grad_cta<THREADS, 4, RECOMPUTE, ENT><<<unsigned(grid_for(1, T)), THREADS, 0, s>>>(
+            logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
     }
 }
 
@@ -239,22 +277,31 @@ using namespace acrl;
 
 extern "C" acrl_status acrl_loss_grad_logits(const acrl_bf16* logits, int64_t T, int64_t V, int64_t ld,
                                              const int32_t* ids, const uint8_t* mask, const float* lse,
-                                             const float* old_logp, const float* coef, float clip_eps,
-                                             acrl_bf16* grad, float* token_loss, float* loss, int32_t* dev_flags,
-                                             acrl_stream stream) {
+                                             const float* old_logp, const float* coef, const float* entropy,
+                                             const float* ent_coef, float clip_eps, acrl_bf16* grad,
+                                             float* token_loss, float* loss, int32_t* dev_flags, acrl_stream stream) {
     if (T < 0 || V < 1 || V > kMaxVocab || ld < V || (ld & 7) != 0) return ACRL_ERR_INVALID_ARG;
     if (!(clip_eps >= 0.f && clip_eps < 1.f)) return ACRL_ERR_INVALID_ARG;
     if (!loss || !dev_flags) return ACRL_ERR_INVALID_ARG;
+    if ((entropy == nullptr) != (ent_coef == nullptr)) return ACRL_ERR_INVALID_ARG;
     if (T > 0 && (!logits || !ids || !coef || !grad || !token_loss)) return ACRL_ERR_INVALID_ARG;
     if (T > 0 && (!aligned16(logits) || !aligned16(grad))) return ACRL_ERR_INVALID_ARG;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     if (T > 0) {
-        if (lse)
-            launch_loss_grad<false>(logits, T, int(V), ld, ids, mask, lse, old_logp, coef, clip_eps, grad, token_loss,
-                                    dev_flags, s);
+        const int v = int(V);
+        const bool ent = ent_coef != nullptr;
+        if (lse && !ent)
+            launch_loss_grad<false, false>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
+                                           clip_eps, grad, token_loss, dev_flags, s);
+        else if (lse && ent)
+            launch_loss_grad<false, true>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
+                                          clip_eps, grad, token_loss, dev_flags, s);
+        else if (!ent)
+            launch_loss_grad<true, false>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
+                                          clip_eps, grad, token_loss, dev_flags, s);
         else
-            launch_loss_grad<true>(logits, T, int(V), ld, ids, mask, lse, old_logp, coef, clip_eps, grad, token_loss,
-                                   dev_flags, s);
+            launch_loss_grad<true, true>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
+                                         clip_eps, grad, token_loss, dev_flags, s);
     }
     loss_sum_kernel<<<1, kSumThreads, 0, s>>>(token_loss, T, loss);
     return launch_status();

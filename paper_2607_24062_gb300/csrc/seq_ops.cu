@@ -238,6 +238,7 @@ __global__ void __launch_bounds__(kFinThreads) controller_alpha_kernel(
     __shared__ int sh_apply;
     if (threadIdx.x == 0) {
         acrl_controller_state s = *st;
+        const bool was_calibrated = s.calibrated != 0;
         int apply = 1;
         if (!s.calibrated) {
             s.calib_sum += batch->Y_sum;
@@ -251,13 +252,17 @@ __global__ void __launch_bounds__(kFinThreads) controller_alpha_kernel(
             }
         }
         s.step += 1;
-        if (p.mode == ACRL_MODE_ACRL && apply && !(s.X > 0.0)) {
+        const bool uses_x = p.mode == ACRL_MODE_ACRL || p.mode == ACRL_MODE_ACRL_FALLBACK;
+        if (uses_x && apply && !(s.X > 0.0)) {
             raise_flag(flags, ACRL_FLAG_X_NONPOS);
             s.flags |= ACRL_FLAG_X_NONPOS;
         }
+        const double X_use = s.X;
+        // moving-average X (off by default): this step uses X_use, the next one the update
+        if (was_calibrated && p.x_ema > 0.f) s.X = (1.0 - double(p.x_ema)) * s.X + double(p.x_ema) * batch->Y_mean;
         *st = s;
-        batch->X = apply ? s.X : 0.0;
-        sh_X = s.X;
+        batch->X = apply ? X_use : 0.0;
+        sh_X = X_use;
         sh_apply = apply;
     }
     __syncthreads();
@@ -266,9 +271,14 @@ __global__ void __launch_bounds__(kFinThreads) controller_alpha_kernel(
     const double Ybatch = batch->Y_mean;
     for (int i = threadIdx.x; i < S; i += kFinThreads) {
         float a = 0.f;
+        const float A = adv[i];
+        const float sgnf = A > 0.f ? 1.f : (A < 0.f ? -1.f : 0.f);
         if (p.mode == ACRL_MODE_TIS || p.mode == ACRL_MODE_MIS) {
             a = 1.f;
-        } else if (p.mode == ACRL_MODE_ACRL && apply && X > 0.0 && seq[i].n > 0) {
+        } else if (p.mode == ACRL_MODE_ACRL_CONTINUOUS) {
+            a = seq[i].n > 0 ? -p.kappa * sgnf : 0.f;
+        } else if ((p.mode == ACRL_MODE_ACRL || p.mode == ACRL_MODE_ACRL_FALLBACK) && apply && X > 0.0 &&
+                   seq[i].n > 0) {
             double Y;
             if (p.y_gran == ACRL_Y_SEQUENCE) {
                 Y = seq[i].sum_d / seq[i].n;
@@ -278,9 +288,8 @@ __global__ void __launch_bounds__(kFinThreads) controller_alpha_kernel(
                 const int g = seq[i].group;
                 Y = (g >= 0 && g < Gn) ? grp[g].Y : 0.0;
             }
-            const float A = adv[i];
-            const double sgn = A > 0.f ? 1.0 : (A < 0.f ? -1.0 : 0.0);
-            a = float(double(p.gamma) * sgn * (1.0 - Y / X));
+            a = float(double(p.gamma) * double(sgnf) * (1.0 - Y / X));
+            if (p.mode == ACRL_MODE_ACRL_FALLBACK && !(Y > X)) a = 0.f;
         }
         seq[i].alpha = a;
         if (alpha_out) alpha_out[i] = a;
@@ -292,7 +301,7 @@ __global__ void __launch_bounds__(kSeqThreads) controller_weights_kernel(
     acrl_params p, const float* __restrict__ lr, const uint8_t* __restrict__ mask, int64_t T,
     const int64_t* __restrict__ so, int Gn, acrl_seq_stats* seq, const acrl_group_stats* __restrict__ grp,
     const acrl_batch_stats* __restrict__ batch, const float* __restrict__ adv, float* __restrict__ weight,
-    float* __restrict__ coef) {
+    float* __restrict__ coef, float* __restrict__ ent_coef) {
     constexpr int NW = kSeqThreads / 32;
     __shared__ double sh_d[NW];
     __shared__ int sh_i[NW];
@@ -309,6 +318,7 @@ __global__ void __launch_bounds__(kSeqThreads) controller_weights_kernel(
         norm = double(batch->n_groups_valid) * double(G) * double(s.n);
     }
     const float scale = norm > 0.0 ? float(double(adv[i]) / norm) : 0.f;
+    const float escale = norm > 0.0 ? float(double(p.entropy_coeff) / norm) : 0.f;
     const float Si = float(s.sum_lr);
     const bool mis_cut = Si > logC;
     const float w_mis = mis_cut ? 0.f : expf(Si);
@@ -332,6 +342,7 @@ __global__ void __launch_bounds__(kSeqThreads) controller_weights_kernel(
         }
         weight[t] = w;
         coef[t] = w * scale;
+        if (ent_coef) ent_coef[t] = m ? escale : 0.f;
     }
     nt = block_sum<int, NW>(nt, sh_i);
     sw = block_sum<double, NW>(sw, sh_d);
@@ -409,8 +420,8 @@ extern "C" acrl_status acrl_controller_step(acrl_controller_state* state, const 
                                             const uint8_t* mask, int64_t T, const int64_t* seq_offsets, int32_t S,
                                             const int32_t* group_offsets, int32_t Gn, acrl_seq_stats* seq,
                                             const acrl_group_stats* grp, acrl_batch_stats* batch, const float* adv,
-                                            float* weight, float* coef, float* alpha, int32_t* dev_flags,
-                                            acrl_stream stream) {
+                                            float* weight, float* coef, float* alpha, float* ent_coef,
+                                            int32_t* dev_flags, acrl_stream stream) {
     if (!state || !params_ok(p) || T < 0 || S < 0 || Gn < 0) return ACRL_ERR_INVALID_ARG;
     if (!seq_offsets || !group_offsets || !batch || !dev_flags) return ACRL_ERR_INVALID_ARG;
     if (T > 0 && (!lr || !weight || !coef)) return ACRL_ERR_INVALID_ARG;
@@ -419,7 +430,7 @@ extern "C" acrl_status acrl_controller_step(acrl_controller_state* state, const 
     controller_alpha_kernel<<<1, kFinThreads, 0, s>>>(state, *p, S, Gn, seq, grp, batch, adv, alpha, dev_flags);
     if (S > 0)
         controller_weights_kernel<<<S, kSeqThreads, 0, s>>>(*p, lr, mask, T, seq_offsets, Gn, seq, grp, batch, adv,
-                                                            weight, coef);
+                                                            weight, coef, ent_coef);
     controller_finalize_kernel<<<1, kFinThreads, 0, s>>>(S, seq, batch);
     return launch_status();
 }

@@ -39,6 +39,7 @@ class AcrlStep:
         self.weight = torch.empty(T, **f32)
         self.coef = torch.empty(T, **f32)
         self.alpha = torch.empty(S, **f32)
+        self.ent_coef = torch.empty(T, **f32) if params.entropy_coeff > 0 else None
         self.grad = torch.empty((grad_rows if grad_rows else T, ld), dtype=torch.bfloat16, device=dev)
         self.token_loss = torch.empty(T, **f32)
         self.loss = torch.empty(1, **f32)
@@ -58,15 +59,18 @@ class AcrlStep:
                             flags=self.flags, stream=stream)
         api.grpo_advantage(rewards, group_offsets, p, adv=self.adv, flags=self.flags, stream=stream)
         api.controller_step(self.state, p, self.disc, mask, seq_offsets, group_offsets, self.adv,
-                            weight=self.weight, coef=self.coef, alpha=self.alpha, flags=self.flags, stream=stream)
+                            weight=self.weight, coef=self.coef, alpha=self.alpha, ent_coef=self.ent_coef,
+                            flags=self.flags, stream=stream)
 
     def gradient(self, logits, ids, mask, stream=None, old_logp=None, recompute_lse=False,
                  chunk_rows: int | None = None, on_chunk: Callable[[int, int, torch.Tensor], None] | None = None):
         """The loss and dL/dlogits (second read of the logits, one write)."""
         lse = None if recompute_lse else self.lse
         eps = self.params.clip_eps
+        ent = self.ent_coef is not None
         if not chunk_rows:
-            api.loss_grad_logits(logits, ids, mask, lse, old_logp, self.coef, eps, V=self.V, grad=self.grad,
+            api.loss_grad_logits(logits, ids, mask, lse, old_logp, self.coef, eps, V=self.V,
+                                 entropy=self.entropy if ent else None, ent_coef=self.ent_coef, grad=self.grad,
                                  token_loss=self.token_loss, loss=self.loss, flags=self.flags, stream=stream)
             return
         for r0 in range(0, self.T, chunk_rows):
@@ -75,6 +79,8 @@ class AcrlStep:
             api.loss_grad_logits(logits[r0:r1], ids[r0:r1], None if mask is None else mask[r0:r1],
                                  None if lse is None else lse[r0:r1],
                                  None if old_logp is None else old_logp[r0:r1], self.coef[r0:r1], eps, V=self.V,
+                                 entropy=self.entropy[r0:r1] if ent else None,
+                                 ent_coef=self.ent_coef[r0:r1] if ent else None,
                                  grad=g, token_loss=self.token_loss[r0:r1], loss=self.chunk_loss, flags=self.flags,
                                  stream=stream)
             if on_chunk is not None:

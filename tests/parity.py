@@ -1,9 +1,13 @@
 """Helpers for comparing the CUDA path (through the C ABI) with the float64
 oracle on the same seeded inputs.  Tolerances are the ones the method's
 arithmetic supports (bf16 in, fp32 accumulation):
-  * log-probs / lse: 2e-4 absolute;
+  * log-probs / lse: 2e-4 absolute; a per-token probability distance d
+    compared with the fp64 chain inherits that bar as |dd| <= pi * 2e-4, and
+    is checked tightly (1e-3 relative) when the oracle is fed the GPU's own
+    fp32 log-probs;
   * entropy, weights, alpha, aggregates, X, batch statistics, loss: 1e-3
-    relative (entropy with a 1e-5 absolute floor);
+    relative (entropy with a 1e-5 absolute floor; the scalar loss with a floor
+    of 1e-6 * sum |token loss|, since the token losses can cancel);
   * bf16 gradient elements: 1e-2 relative; an element whose reference is
     below 2^-125 may come back as 0 (the exp2 flushes subnormals); the
     sampled column, coef * (p_a - 1), carries the fp32 error of logp_a, so it
@@ -29,6 +33,7 @@ def host(t):
 
 def oracle_params(p) -> O.Params:
     return O.Params(gamma=float(p.gamma), C=float(p.C), clip_eps=float(p.clip_eps), adv_eps=float(p.adv_eps),
+                    kappa=float(p.kappa), x_ema=float(p.x_ema), entropy_coeff=float(p.entropy_coeff),
                     mode=int(p.mode), y_gran=int(p.y_gran), agg=int(p.agg), adv_ddof=int(p.adv_ddof),
                     singleton_rule=int(p.singleton_rule), calib_steps=int(p.calib_steps), X_init=float(p.X_init))
 
@@ -67,12 +72,16 @@ def assert_close_abs(got, ref, tol, what=""):
                              f"ref {ref.ravel()[k]} at {k}")
 
 
-def assert_grad_rows(got, ref, coef_eff, ids_rows, what="grad"):
-    """got/ref [R, V]; coef_eff [R] = the reference coef_t g_t r_t."""
+def assert_grad_rows(got, ref, coef_eff, ids_rows, what="grad", row_floor=0.0):
+    """got/ref [R, V]; coef_eff [R] = the reference coef_t g_t r_t.  With an
+    entropy bonus an element is p_j (c + e (z_j - lse + H)), whose bracket can
+    cancel; `row_floor` then adds row_floor * max_j |ref[t, j]| per row."""
     got = np.asarray(got, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
     tol = TOL_GRAD * np.abs(ref)
     tol = np.maximum(tol, np.where(np.abs(ref) < FTZ, FTZ, 0.0))
+    if row_floor:
+        tol += row_floor * np.abs(ref).max(axis=1, keepdims=True)
     R = ref.shape[0]
     cols = np.asarray(ids_rows, dtype=np.int64)
     ok_ids = (cols >= 0) & (cols < ref.shape[1])

@@ -29,8 +29,8 @@ def test_exports_every_declared_function(L):
 
 
 def test_abi_version_and_layouts(L):
-    assert L.acrl_abi_version() == 1
-    assert L.acrl_struct_size(0) == ctypes.sizeof(_abi.Params) == 48
+    assert L.acrl_abi_version() == 2
+    assert L.acrl_struct_size(0) == ctypes.sizeof(_abi.Params) == 64
     assert L.acrl_struct_size(1) == 48 and L.acrl_struct_size(2) == 64
     assert L.acrl_struct_size(3) == 24 and L.acrl_struct_size(4) == 104
     assert L.acrl_struct_size(99) == -1
@@ -57,10 +57,16 @@ def test_host_side_rejections(L):
     assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(calib_steps=0)), None) == E
     assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(mode=7)), None) == E
     # loss/grad: clip eps out of range, misaligned grad
-    assert L.acrl_loss_grad_logits(fake, 4, 16, 16, fake, None, None, None, fake, 1.5, fake, fake, fake, fake,
-                                   None) == E
-    assert L.acrl_loss_grad_logits(fake, 4, 16, 16, fake, None, None, None, fake, 0.2, fake + 8, fake, fake, fake,
-                                   None) == E
+    assert L.acrl_loss_grad_logits(fake, 4, 16, 16, fake, None, None, None, fake, None, None, 1.5, fake, fake, fake,
+                                   fake, None) == E
+    assert L.acrl_loss_grad_logits(fake, 4, 16, 16, fake, None, None, None, fake, None, None, 0.2, fake + 8, fake,
+                                   fake, fake, None) == E
+    # the entropy bonus needs both the entropies and their coefficients
+    assert L.acrl_loss_grad_logits(fake, 4, 16, 16, fake, None, None, None, fake, fake, None, 0.2, fake, fake, fake,
+                                   fake, None) == E
+    assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(kappa=0.0)), None) == E
+    assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(x_ema=1.5)), None) == E
+    assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(entropy_coeff=-1.0)), None) == E
     assert L.acrl_read_flags(None, None, None) == E
     assert L.acrl_reduce_loss(None, 4, fake, None) == E
 

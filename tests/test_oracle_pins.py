@@ -391,14 +391,18 @@ def _torch_loss(zt, f, params):
             A = f["adv"][i]
             surr = torch.minimum(r[t] * A, torch.clamp(r[t], 1 - params.clip_eps, 1 + params.clip_eps) * A)
             total = total - f["w"][t] * surr / norm
+            if params.entropy_coeff:
+                ent = -(torch.softmax(zt[t], 0) * logq[t]).sum()
+                total = total - params.entropy_coeff * ent / norm
     return total
 
 
+@pytest.mark.parametrize("beta", [0.0, 0.05])
 @pytest.mark.parametrize("with_old", [False, True])
-def test_gradient_matches_autograd(with_old):
+def test_gradient_matches_autograd(with_old, beta):
     rng = np.random.default_rng(21 + with_old)
     f = _fixture(rng, with_old=with_old)
-    p = O.Params()
+    p = O.Params(entropy_coeff=beta)
     grad, tl, loss = O.loss_grad_logits(f["z"], f["ids"], f["mask"], None, f["old"], f["adv"], f["w"], f["so"],
                                         f["seq"], f["grp"], f["batch"], p)
     zt = torch.tensor(f["z"], dtype=torch.float64, requires_grad=True)
@@ -408,10 +412,11 @@ def test_gradient_matches_autograd(with_old):
     assert loss == pytest.approx(float(L), abs=1e-14)
 
 
-def test_gradient_central_differences():
+@pytest.mark.parametrize("beta", [0.0, 0.3])
+def test_gradient_central_differences(beta):
     rng = np.random.default_rng(33)
     f = _fixture(rng, V=6, with_old=True)
-    p = O.Params()
+    p = O.Params(entropy_coeff=beta)
 
     def L(z):
         return O.loss_grad_logits(z, f["ids"], f["mask"], None, f["old"], f["adv"], f["w"], f["so"], f["seq"],
@@ -504,3 +509,74 @@ def test_coefficients_and_surrogate_agree_with_gradient(with_old):
         pr = np.exp(f["z"][t] - lse[t])
         pr[f["ids"][t]] -= 1.0
         np.testing.assert_allclose(grad[t], coef[t] * r * gate * pr, atol=1e-15)
+
+
+def test_entropy_bonus_by_hand():
+    # uniform rows: H = ln V, so each valid token adds -beta ln V / norm to the loss
+    V = 6
+    z = np.zeros((3, V))
+    ids = np.array([0, 1, 2])
+    seq = {"n": np.array([2, 1]), "group": np.array([0, 0])}
+    grp = {"n_valid_seqs": np.array([2])}
+    batch = {"n_groups_valid": 1, "n_tokens": 3}
+    adv = np.array([0.0, 0.0])                     # no policy term: only the bonus
+    p = O.Params(entropy_coeff=0.1)
+    grad, tl, loss = O.loss_grad_logits(z, ids, None, None, None, adv, np.ones(3), [0, 2, 3], seq, grp, batch, p)
+    assert loss == pytest.approx(-0.1 * math.log(V) * (1 / 4 + 1 / 4 + 1 / 2), abs=1e-15)
+    # at the uniform distribution the entropy is maximal: its gradient vanishes
+    np.testing.assert_allclose(grad, 0.0, atol=1e-16)
+    beta_t = O.entropy_coefficients(None, [0, 2, 3], seq, grp, batch, p)
+    np.testing.assert_allclose(beta_t, [0.1 / 4, 0.1 / 4, 0.1 / 2], rtol=1e-15)
+
+
+@pytest.mark.parametrize("row", _read_quadrants(), ids=lambda r: f"{r[0]}-{r[1]}")
+def test_continuous_reduction_always_reduces(row):
+    # Sec. 5.5: alpha = -1 where A > 0 and +1 where A < 0 whatever Y and X are, so every
+    # quadrant follows the Y > X (decrease) row of the sign table.
+    _, quad, sA, pvm = row[:4]
+    table = {r[1]: r for r in _read_quadrants() if r[0] == "Y>X"}
+    A = 1.0 if sA == "+" else -1.0
+    pi, mu = (0.3, 0.5) if pvm == "<" else (0.5, 0.3)
+    for Y in (0.005, 0.02):
+        w, alpha, *_ = _one_token_case(pi, mu, A, Y, 0.013, mode=O.MODE_ACRL_CONTINUOUS)
+        assert alpha[0] == -A
+        assert (w[0] > 1) == (table[quad][5] == ">")
+        assert w[0] == pytest.approx(min((pi / mu) ** -A, 3.0), rel=1e-14)
+
+
+def test_continuous_reduction_kappa():
+    w, alpha, *_ = _one_token_case(0.2, 0.4, -1.0, 0.0, 0.013, mode=O.MODE_ACRL_CONTINUOUS)
+    assert alpha[0] == 1.0 and w[0] == pytest.approx(0.5, rel=1e-14)
+    p = O.Params(mode=O.MODE_ACRL_CONTINUOUS, kappa=3.0, X_init=0.013)
+    lr = np.array([math.log(0.5)])
+    seq = {"n": np.array([1]), "group": np.array([0]), "mean_d": np.array([0.0]), "sum_lr": lr}
+    grp = {"Y": np.array([0.0]), "n_valid_seqs": np.array([1])}
+    batch = {"Y_sum": 0.0, "Y_mean": 0.0, "n_groups_valid": 1}
+    w, alpha, *_ = O.controller_step(O.controller_init(p), p, lr, None, [0, 1], [0, 1], seq, grp, batch, [2.0])
+    assert alpha[0] == -3.0 and w[0] == pytest.approx(3.0, rel=1e-14)   # (1/2)^-3 = 8, truncated at C = 3
+
+
+def test_fallback_to_grpo():
+    # Y < X: plain GRPO (w = 1); Y > X: the ACRL weight
+    w, alpha, *_ = _one_token_case(0.2, 0.4, 1.0, 0.005, 0.013, mode=O.MODE_ACRL_FALLBACK)
+    assert alpha[0] == 0.0 and w[0] == 1.0
+    w, alpha, *_ = _one_token_case(0.2, 0.4, 1.0, 0.026, 0.013, mode=O.MODE_ACRL_FALLBACK, gamma=0.5)
+    assert alpha[0] == pytest.approx(-0.5, abs=1e-15) and w[0] == pytest.approx(math.sqrt(2), rel=1e-14)
+
+
+def test_moving_average_X_by_hand():
+    # X frozen by default; with x_ema = 0.5 each later step moves X halfway to that step's Y
+    p = O.Params(x_ema=0.5)
+    st = O.controller_init(p)
+    Xs = []
+    for Y in (0.02, 0.04, 0.01):
+        lr = np.array([0.1])
+        seq = {"n": np.array([1]), "group": np.array([0]), "mean_d": np.array([Y]), "sum_lr": lr}
+        grp = {"Y": np.array([Y]), "n_valid_seqs": np.array([1])}
+        batch = {"Y_sum": Y, "Y_mean": Y, "n_groups_valid": 1}
+        _, _, st, info, _ = O.controller_step(st, p, lr, None, [0, 1], [0, 1], seq, grp, batch, [1.0])
+        Xs.append((info["X"], st.X))
+    # step 0 calibrates X = 0.02 (no update on that step); step 1 uses 0.02 then moves to 0.03; step 2 uses 0.03
+    assert Xs[0] == (pytest.approx(0.02), pytest.approx(0.02))
+    assert Xs[1] == (pytest.approx(0.02), pytest.approx(0.03))
+    assert Xs[2] == (pytest.approx(0.03), pytest.approx(0.02))

@@ -80,7 +80,8 @@ def _full_chain_check(b, params, state=None):
     # a6
     assert_close_rel(host(step.token_loss), res.token_loss, floor=1e-12, what="token_loss")
     assert_loss(float(step.loss), res.loss, res.token_loss)
-    assert_grad_rows(grad_rows(step.grad, np.arange(b.T), b.V), res.grad, coef_ref, h["ids"])
+    assert_grad_rows(grad_rows(step.grad, np.arange(b.T), b.V), res.grad, coef_ref, h["ids"],
+                     row_floor=1e-6 if op.entropy_coeff else 0.0)
     flags = api.read_flags(step.flags)
     assert flags == res.flags, (flags, res.flags)
     return step, res
@@ -132,18 +133,21 @@ def test_empty_sequence_and_group():
     assert res.batch["n_groups_valid"] == 2
 
 
-@pytest.mark.parametrize("mode", [acrl.MODE_NONE, acrl.MODE_TIS, acrl.MODE_MIS, acrl.MODE_ACRL])
+@pytest.mark.parametrize("mode", [acrl.MODE_NONE, acrl.MODE_TIS, acrl.MODE_MIS, acrl.MODE_ACRL,
+                                  acrl.MODE_ACRL_CONTINUOUS, acrl.MODE_ACRL_FALLBACK])
 @pytest.mark.parametrize("y_gran", [acrl.Y_GROUP, acrl.Y_SEQUENCE, acrl.Y_BATCH])
 def test_modes(mode, y_gran):
-    if mode != acrl.MODE_ACRL and y_gran != acrl.Y_GROUP:
-        pytest.skip("y granularity only matters for ACRL")
+    if mode not in (acrl.MODE_ACRL, acrl.MODE_ACRL_FALLBACK) and y_gran != acrl.Y_GROUP:
+        pytest.skip("y granularity only matters for the modes that compare Y with X")
     spec = W.small_variant(W.QWEN, name="modes", n_prompts=3, group_size=4, len_lo=4, len_hi=60, V=2048,
                            perturb_frac=0.5, perturb_std=0.3)
     _full_chain_check(_gen(spec, seed=77), acrl.Params(mode=mode, y_gran=y_gran, gamma=1.3, C=5.0))
 
 
 @pytest.mark.parametrize("kw", [dict(agg=acrl.AGG_TOKEN_MEAN), dict(adv_ddof=0), dict(X_init=0.013),
-                                dict(singleton_rule=acrl.SINGLETON_ZERO), dict(calib_steps=2)])
+                                dict(singleton_rule=acrl.SINGLETON_ZERO), dict(calib_steps=2),
+                                dict(entropy_coeff=0.001), dict(entropy_coeff=0.05, agg=acrl.AGG_TOKEN_MEAN),
+                                dict(X_init=0.013, x_ema=0.3), dict(mode=acrl.MODE_ACRL_CONTINUOUS, kappa=3.0)])
 def test_param_options(kw):
     spec = W.small_variant(W.TINY, name="opts", n_prompts=3, group_size=2, len_lo=20, len_hi=70, V=1000)
     _full_chain_check(_gen(spec, seed=5), acrl.Params(**kw))
@@ -177,21 +181,26 @@ def test_uniform_logits_and_equal_policies():
     assert api.read_flags(flags) == acrl.FLAG_X_NONPOS
 
 
-def test_old_logp_and_recomputed_lse():
-    """Cached-old path: weights from old log-probs, LSE recomputed in the gradient kernel, r != 1 with clipping."""
-    spec = W.small_variant(W.QWEN, name="offpolicy", n_prompts=2, group_size=4, len_lo=10, len_hi=80, V=20011)
+@pytest.mark.parametrize("beta", [0.0, 0.01])
+@pytest.mark.parametrize("V", [20011, 4099])
+def test_old_logp_and_recomputed_lse(V, beta):
+    """Cached-old path: weights from old log-probs, LSE recomputed in the gradient kernel, r != 1 with clipping
+    (CTA and warp row teams, with and without the entropy bonus)."""
+    spec = W.small_variant(W.QWEN, name="offpolicy", n_prompts=2, group_size=4, len_lo=10, len_hi=80, V=V)
     b = _gen(spec, seed=31)
-    p = acrl.Params()
+    p = acrl.Params(entropy_coeff=beta)
     gen = torch.Generator(device=DEV).manual_seed(3)
     lse, logp, H = api.token_stats(b.logits, b.ids, b.mask, V=b.V)
     old = (logp + 0.3 * torch.randn(b.T, generator=gen, device=DEV)).clamp(max=0.0)
     disc = api.seq_discrepancy(old, b.logp_mu, b.mask, b.seq_offsets, b.group_offsets, H)
     adv = api.grpo_advantage(b.rewards, b.group_offsets, p)
     state = api.controller_init(p)
-    w, coef, alpha = api.controller_step(state, p, disc, b.mask, b.seq_offsets, b.group_offsets, adv)
+    ent_coef = torch.empty(b.T, device=DEV) if beta else None
+    w, coef, alpha = api.controller_step(state, p, disc, b.mask, b.seq_offsets, b.group_offsets, adv,
+                                         ent_coef=ent_coef)
     for recompute in (False, True):
         grad, tl, loss = api.loss_grad_logits(b.logits, b.ids, b.mask, None if recompute else lse, old, coef,
-                                              p.clip_eps, V=b.V)
+                                              p.clip_eps, V=b.V, entropy=H if beta else None, ent_coef=ent_coef)
         torch.cuda.synchronize()
         h = _host_inputs(b)
         op = oracle_params(p)
@@ -206,10 +215,15 @@ def test_old_logp_and_recomputed_lse():
         ograd, otl, oloss = O.loss_grad_logits(z, h["ids"], h["mask"], None, oold, oadv, ow, h["so"], seq, grp,
                                                batch, op)
         coef_ref = O.loss_coefficients(ow, oadv, h["mask"], h["so"], seq, grp, batch, op)
+        if beta:
+            ecoef = O.entropy_coefficients(h["mask"], h["so"], seq, grp, batch, op)
+            assert_close_rel(host(ent_coef), ecoef, floor=1e-12, what="ent_coef")
         r = np.exp(ologp - oold)
         gate = np.where(coef_ref >= 0, r <= 1 + op.clip_eps, r >= 1 - op.clip_eps)
         assert 0 < gate.sum() < len(gate)   # both branches exercised
-        assert_grad_rows(grad_rows(grad, np.arange(b.T), b.V), ograd, coef_ref * r * gate, h["ids"])
+        # the sampled column's absolute floor scales with the largest coefficient on the row
+        scale = np.abs(coef_ref * r * gate) + (ecoef * (1 + np.abs(oH)) if beta else 0.0)
+        assert_grad_rows(grad_rows(grad, np.arange(b.T), b.V), ograd, scale, h["ids"], row_floor=1e-6 if beta else 0)
         assert_close_rel(host(tl), otl, floor=1e-12, what="token_loss")
         assert_loss(float(loss), oloss, otl)
 
