@@ -41,7 +41,12 @@ LAUNCHES_PER_STEP = 9
 # DRAM traffic of one gradient-kernel launch on the bench workload, from ncu
 # (dram__bytes_read.sum + dram__bytes_write.sum), valid only for the kernel source
 # it was taken on (sha256 of the file, first 16 hex digits).
-NCU_TRAFFIC = {}
+# Taken with `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` (one pass) on the
+# bench workload; see profiles/dram_traffic_qwen_bench.md.
+NCU_TRAFFIC = {
+    "loss_grad.cu": {"src": "0a208a2210e7f12c", "bytes_per_launch": 41.71e9 + 44.87e9},
+    "token_stats.cu": {"src": "4c54a894cb214469", "bytes_per_launch": 44.93e9 + 3.45e6},
+}
 
 
 def _peaks():
@@ -312,8 +317,10 @@ def run_ours(args):
     k1_avg = float(np.mean(k1_ms))
     k5_gbs = k5_bytes / (k5_avg / 1e3) / 1e9
     k1_gbs = k1_bytes / (k1_avg / 1e3) / 1e9
-    tr = NCU_TRAFFIC.get("loss_grad.cu")
-    traffic = tr["bytes_per_launch"] if tr and tr["src"] == _src_hash("loss_grad.cu") else None
+    def traffic_of(name):
+        tr = NCU_TRAFFIC.get(name)
+        return tr["bytes_per_launch"] if tr and tr["src"] == _src_hash(name) else None
+    traffic = traffic_of("loss_grad.cu")
 
     e2e = None
     if not args.no_e2e and rank == 0:
@@ -334,7 +341,8 @@ def run_ours(args):
                      "unit": "GB/s", "frac": k5_gbs / peak, "traffic": traffic, "peak_kind": peak_kind,
                      "algorithmic_bytes_per_launch": k5_bytes, "ms_per_launch": k5_avg},
         "kernels": {
-            "acrl_token_stats": {"ms": k1_avg, "GB/s": k1_gbs, "frac": k1_gbs / peak, "bytes": k1_bytes},
+            "acrl_token_stats": {"ms": k1_avg, "GB/s": k1_gbs, "frac": k1_gbs / peak, "bytes": k1_bytes,
+                                 "traffic": traffic_of("token_stats.cu")},
             "acrl_loss_grad_logits": {"ms": k5_avg, "GB/s": k5_gbs, "frac": k5_gbs / peak, "bytes": k5_bytes},
             "seq_discrepancy+grpo_advantage+controller_step": {"ms": float(np.mean(mid_ms))},
             "whole_step_GB/s": (k1_bytes + k5_bytes) / (ms_per_step / 1e3) / 1e9,
@@ -355,9 +363,9 @@ def run_e2e(batch, step, params, args, dev):
     """Same metric through the public API with the user's buffers in host
     memory: every step uploads that step's inputs from page-locked host memory,
     runs the whole path and downloads the gradient and the loss.  Rows move in
-    chunks on two copy streams so that uploads overlap the statistics kernel,
-    downloads overlap the gradient kernel, and one step's downloads overlap the
-    next step's uploads; events order every reuse of a device or host chunk."""
+    chunks on a copy stream so that uploads overlap the statistics kernel and
+    downloads overlap the gradient kernel; events order every reuse of a
+    device or host chunk."""
     import torch
 
     import paper_2607_24062_gb300 as acrl
@@ -384,7 +392,10 @@ def run_e2e(batch, step, params, args, dev):
         loss_h = torch.empty(1, dtype=torch.float32, pin_memory=True)
         d_logits = batch.logits
         comp = torch.cuda.current_stream(dev)
-        s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        # Both directions share one copy stream: on this link a download running at the same time as an
+        # upload slowed the pair to a fraction of either alone, so the copies are kept one-way at a time
+        # while the kernels overlap them.
+        s_in = s_out = torch.cuda.Stream(dev)
         nchunk = max(1, args.e2e_chunks)
         bounds = [(T * k // nchunk, T * (k + 1) // nchunk) for k in range(nchunk)]
         E = torch.cuda.Event
