@@ -58,6 +58,8 @@ typedef enum {
 #define ACRL_FLAG_NONFINITE   0x2   /* a valid row held a NaN or an infinity   */
 #define ACRL_FLAG_BAD_OFFSETS 0x4   /* seq/group offsets not monotone or not covering */
 #define ACRL_FLAG_X_NONPOS    0x8   /* ACRL mode with a reference X <= 0       */
+#define ACRL_FLAG_TIMEOUT     0x10  /* a pipeline wait inside the tensor-core kernel gave
+                                       up after its time limit: that call's outputs are invalid */
 
 /* Importance-weight mode. */
 typedef enum {
@@ -323,6 +325,40 @@ acrl_status acrl_loss_grad_logits(const acrl_bf16* logits, int64_t T, int64_t V,
  *   token_loss  device float [T];  loss  device float [1] output.
  */
 acrl_status acrl_reduce_loss(const float* token_loss, int64_t T, float* loss, acrl_stream stream);
+
+/*
+ * acrl_lmhead_logits_stats -- the LM-head projection logits = H W^T fused
+ * with the log-softmax statistics of acrl_token_stats (the optional fused
+ * path of the logits pass; the paper's policy pi ends in this projection).
+ * bf16 inputs, fp32 accumulation on the tensor cores (tcgen05, TMEM), logits
+ * rounded to bf16 and stored; for every row and every 256-column tile the
+ * epilogue writes the online state (max, U = max log2e, sum 2^(u-U),
+ * sum 2^(u-U)(u-U)) of those bf16 logits to `partials`, which
+ * acrl_lmhead_merge turns into lse / logp / entropy.
+ *   hidden   device bf16 [M, ldh] (K used), weight device bf16 [N, ldw] (K used),
+ *            both 16-byte aligned with ldh, ldw multiples of 8.
+ *   logits   device bf16 [M, ldl] output (ldl >= N, multiple of 8).
+ *   partials device float4 workspace of acrl_lmhead_workspace_bytes(M, N)
+ *            bytes, layout [ceil(N/256)][M]; owned by the caller.
+ * Pipeline waits are time-bounded: ACRL_FLAG_TIMEOUT means the outputs of this
+ * call are invalid.  Requires an sm_100-family GPU (built for sm_103a).
+ */
+int64_t     acrl_lmhead_workspace_bytes(int64_t M, int64_t N);
+acrl_status acrl_lmhead_logits_stats(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t ldh,
+                                     const acrl_bf16* weight, int64_t N, int64_t ldw,
+                                     acrl_bf16* logits, int64_t ldl, float* partials,
+                                     int32_t* dev_flags, acrl_stream stream);
+
+/*
+ * acrl_lmhead_merge -- lse, logp = z[a] - lse and entropy per row from the
+ * partial states of acrl_lmhead_logits_stats (tiles merged in order, so the
+ * result is deterministic); same outputs, masking and flags as
+ * acrl_token_stats.  z[a] is read from `logits`.
+ */
+acrl_status acrl_lmhead_merge(const float* partials, const acrl_bf16* logits, int64_t M, int64_t N,
+                              int64_t ldl, const int32_t* ids, const uint8_t* mask,
+                              float* lse, float* logp, float* entropy,
+                              int32_t* dev_flags, acrl_stream stream);
 
 /* Copy the device flags word to *host_flags; synchronises `stream`. */
 acrl_status acrl_read_flags(const int32_t* dev_flags, int32_t* host_flags, acrl_stream stream);

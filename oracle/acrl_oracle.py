@@ -122,6 +122,25 @@ def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
     return u.view(np.float32).astype(np.float64)
 
 
+def round_bf16(x) -> np.ndarray:
+    """Round float64 values to the nearest bf16 value, ties to even (8
+    significant bits), returned as float64.  Written from the format's
+    definition: x = f 2^e with f in [0.5, 1); keep f to 8 bits with
+    round-half-even.  Finite normal range only (logits)."""
+    x = np.asarray(x, dtype=np.float64)
+    f, e = np.frexp(x)
+    return np.ldexp(np.rint(f * 256.0) / 256.0, e)
+
+
+def lmhead_logits(hidden, weight) -> np.ndarray:
+    """The policy's logits z = H W^T of an LM-head projection, with the
+    products summed exactly enough in float64 and the result stored in bf16
+    (the training engine's bf16 logits).  hidden [R, K], weight [N, K]."""
+    H = np.asarray(hidden, dtype=np.float64)
+    Wt = np.asarray(weight, dtype=np.float64)
+    return round_bf16(H @ Wt.T)
+
+
 # --------------------------------------------------------------------------
 # a1: log-softmax, sampled-token log-prob, entropy
 # --------------------------------------------------------------------------

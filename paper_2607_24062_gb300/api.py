@@ -213,6 +213,54 @@ def reduce_loss(token_loss, *, loss=None, stream=None):
     return loss
 
 
+def lmhead_workspace_bytes(M: int, N: int) -> int:
+    return int(lib().acrl_lmhead_workspace_bytes(M, N))
+
+
+def lmhead_logits_stats(hidden, weight, *, N=None, logits=None, partials=None, flags=None, stream=None):
+    """acrl_lmhead_logits_stats.  hidden bf16 [M, K], weight bf16 [N, K].
+    Returns (logits bf16 [M, ldl], partials workspace)."""
+    M, ldh = _rows(hidden, "hidden")
+    Nw, ldw = _rows(weight, "weight")
+    N = Nw if N is None else N
+    K = hidden.shape[1]
+    if weight.shape[1] != K:
+        raise AcrlError("hidden and weight disagree on K")
+    dev = hidden.device
+    ldl = ((N + 7) // 8) * 8
+    if logits is None:
+        logits = torch.empty((M, ldl), dtype=torch.bfloat16, device=dev)
+    else:
+        _, ldl = _rows(logits, "logits")
+    nbytes = lmhead_workspace_bytes(M, N)
+    if partials is None:
+        partials = torch.empty(max(1, nbytes // 4), dtype=torch.float32, device=dev)
+    elif partials.numel() * 4 < nbytes:
+        raise AcrlError("partials: workspace too small")
+    flags = new_flags(dev) if flags is None else flags
+    check(lib().acrl_lmhead_logits_stats(_ptr(hidden), M, K, ldh, _ptr(weight), N, ldw, _ptr(logits), ldl,
+                                         _ptr(partials), _ptr(flags), _stream(stream)), "acrl_lmhead_logits_stats")
+    return logits, partials
+
+
+def lmhead_merge(partials, logits, ids, mask=None, *, N=None, lse=None, logp=None, entropy=None, flags=None,
+                 stream=None):
+    """acrl_lmhead_merge.  Returns (lse, logp, entropy)."""
+    M, ldl = _rows(logits, "logits")
+    N = ldl if N is None else N
+    dev = logits.device
+    _need(ids, torch.int32, M, "ids")
+    _opt(mask, torch.uint8, M, "mask")
+    lse = torch.empty(M, dtype=torch.float32, device=dev) if lse is None else _need(lse, torch.float32, M, "lse")
+    logp = torch.empty(M, dtype=torch.float32, device=dev) if logp is None else _need(logp, torch.float32, M, "logp")
+    entropy = torch.empty(M, dtype=torch.float32, device=dev) if entropy is None else \
+        _need(entropy, torch.float32, M, "entropy")
+    flags = new_flags(dev) if flags is None else flags
+    check(lib().acrl_lmhead_merge(_ptr(partials), _ptr(logits), M, N, ldl, _ptr(ids), _ptr(mask), _ptr(lse),
+                                  _ptr(logp), _ptr(entropy), _ptr(flags), _stream(stream)), "acrl_lmhead_merge")
+    return lse, logp, entropy
+
+
 def read_flags(flags, stream=None) -> int:
     """acrl_read_flags (synchronises the stream)."""
     host = ctypes.c_int32(0)
@@ -222,4 +270,5 @@ def read_flags(flags, stream=None) -> int:
 
 __all__ = ["Params", "AcrlError", "token_stats", "seq_discrepancy", "grpo_advantage", "controller_init",
            "controller_step", "loss_grad_logits", "reduce_loss", "read_flags", "read_state", "Discrepancy",
+           "lmhead_logits_stats", "lmhead_merge", "lmhead_workspace_bytes",
            "struct_buffer", "read_structs", "new_flags", "_abi"]

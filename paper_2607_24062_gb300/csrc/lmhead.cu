@@ -1,0 +1,452 @@
+// LM-head projection on the tensor cores with the log-softmax statistics in
+// the epilogue: logits = H W^T (bf16 inputs, fp32 accumulation, bf16 output),
+// and for every (row, 256-column tile) the online state (max, sum 2^(u-U),
+// sum 2^(u-U)(u-U)) of the bf16-rounded logits, so that the merge kernel gets
+// lse, the sampled token's log-prob and the entropy without reading the logits
+// again.
+//
+// Blackwell path: a persistent kernel, one CTA per SM, warp-specialised.
+//   warp 0     one thread issues TMA tile loads (128B-swizzled) into a 4-stage
+//              shared-memory ring (A 128x64 + B 256x64 bf16 per stage);
+//   warp 1     one thread issues tcgen05.mma (M=128, N=256, K=16, kind::f16)
+//              into a TMEM accumulator and commits each stage back to the
+//              producer; two 256-column accumulators alternate between tiles;
+//   warps 2-5  the epilogue: tcgen05.ld of the accumulator (each thread one
+//              row), round to bf16, store the logits, fold the statistics.
+// Tiles are visited in bands of 16 row tiles so that the weight tiles in
+// flight are shared through L2 by the CTAs working on the same band.
+// Every wait on an mbarrier is bounded in time; on expiry the kernel raises
+// ACRL_FLAG_TIMEOUT, lets the copies it issued land, and exits after freeing
+// its TMEM.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "acrl_device.cuh"
+#include "acrl_host.h"
+#include "row_lse.cuh"
+
+namespace acrl {
+namespace {
+
+constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
+constexpr int kABytes = kBM * kBK * 2;
+constexpr int kBBytes = kBN * kBK * 2;
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 512;
+constexpr int kBandM = 16;
+constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s: every legitimate wait is microseconds
+// Instruction descriptor of tcgen05.mma kind::f16: D f32 (bits 4-5 = 1),
+// A and B bf16 (bits 7-9, 10-12 = 1), both K-major, N/8 at bit 17, M/16 at bit 24.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kBN >> 3) << 17) |
+                            (uint32_t(kBM >> 4) << 24);
+
+struct Barriers {
+    uint64_t full[kStages];
+    uint64_t empty[kStages];
+    uint64_t tfull[2];
+    uint64_t tempty[2];
+    uint64_t mma_done;
+    uint32_t tmem_base;
+    int32_t abort;
+};
+
+constexpr int kSmemBytes = 1024 + kStages * kStageBytes + int(sizeof(Barriers));
+
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Wait for the completion of the phase of `bar` with parity `parity`.  Gives
+// up after kWaitNs, or early once another role has set *abort (unless abort
+// is null).
+__device__ __noinline__ bool wait_phase(uint64_t* bar, uint32_t parity, volatile int32_t* abort) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 255u) == 0u) {
+            if (abort && *abort) return false;
+            if (global_ns() - t0 > kWaitNs) return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with
+// 128-byte swizzling: rows of 128 bytes, 8-row groups 1024 bytes apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
+    uint64_t d = uint64_t((addr & 0x3FFFFu) >> 4);  // start address
+    d |= uint64_t(1024 >> 4) << 32;                  // stride between 8-row groups
+    d |= uint64_t(1) << 46;                          // descriptor version of tcgen05
+    d |= uint64_t(2) << 61;                          // 128-byte swizzle
+    return d;
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+            tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
+        "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+          "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// ---------------------------------------------------------------------------
+// tile schedule: bands of kBandM row tiles, all column tiles of a band in turn
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ void tile_coords(int t, int m_tiles, int n_tiles, int& m, int& n) {
+    const int per_band = kBandM * n_tiles;
+    const int band = t / per_band;
+    const int r = t - band * per_band;
+    const int bm = min(kBandM, m_tiles - band * kBandM);
+    m = band * kBandM + r % bm;
+    n = r / bm;
+}
+
+__device__ __forceinline__ void give_up(volatile int32_t* abort, int32_t* flags) {
+    *abort = 1;
+    raise_flag(flags, ACRL_FLAG_TIMEOUT);
+}
+
+// ---------------------------------------------------------------------------
+// roles
+// ---------------------------------------------------------------------------
+
+__device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t* sA, uint8_t* sB, Barriers* bars,
+                         int m_tiles, int n_tiles, int total, int k_iters, int32_t* flags) {
+    volatile int32_t* abort = &bars->abort;
+    int stage = 0;
+    uint32_t phase = 0;
+    long issued = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+        int m, n;
+        tile_coords(t, m_tiles, n_tiles, m, n);
+        for (int kk = 0; kk < k_iters; ++kk) {
+            if (!wait_phase(&bars->empty[stage], phase ^ 1u, abort)) {
+                give_up(abort, flags);
+                ok = false;
+                break;
+            }
+            mbar_expect_tx(&bars->full[stage], kStageBytes);
+            tma_load_2d(sA + stage * kABytes, tmA, &bars->full[stage], kk * kBK, m * kBM);
+            tma_load_2d(sB + stage * kBBytes, tmB, &bars->full[stage], kk * kBK, n * kBN);
+            ++issued;
+            if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+    }
+    if (!ok) {
+        // let the copies this thread started land before the CTA can exit
+        for (long j = issued - 1; j >= 0 && j >= issued - kStages; --j)
+            wait_phase(&bars->full[j % kStages], uint32_t((j / kStages) & 1), nullptr);
+    }
+}
+
+__device__ void mma_issuer(uint8_t* sA, uint8_t* sB, Barriers* bars, uint32_t tmem, int total, int k_iters,
+                           int32_t* flags) {
+    volatile int32_t* abort = &bars->abort;
+    int stage = 0;
+    uint32_t phase = 0;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+        if (!wait_phase(&bars->tempty[acc], acc_phase ^ 1u, abort)) {
+            give_up(abort, flags);
+            break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + uint32_t(acc * kBN);
+        for (int kk = 0; kk < k_iters; ++kk) {
+            if (!wait_phase(&bars->full[stage], phase, abort)) {
+                give_up(abort, flags);
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t a0 = smem_u32(sA + stage * kABytes);
+            const uint32_t b0 = smem_u32(sB + stage * kBBytes);
+#pragma unroll
+            for (int k16 = 0; k16 < kBK / 16; ++k16)
+                mma_bf16(d, sw128_desc(a0 + k16 * 32), sw128_desc(b0 + k16 * 32), (kk | k16) != 0);
+            mma_commit(&bars->empty[stage]);
+            if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+        if (!ok) break;
+        mma_commit(&bars->tfull[acc]);
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+    }
+    // every MMA this thread issued has finished before the CTA moves on
+    mma_commit(&bars->mma_done);
+    wait_phase(&bars->mma_done, 0, nullptr);
+}
+
+__device__ void epilogue(Barriers* bars, uint32_t tmem, int M, int N, int m_tiles, int n_tiles, int total,
+                         acrl_bf16* __restrict__ logits, int64_t ldl, float4* __restrict__ partials, int32_t* flags) {
+    volatile int32_t* abort = &bars->abort;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int quarter = warp & 3;  // the TMEM lanes (rows) this warp may read
+    const uint32_t lane_off = uint32_t(quarter * 32) << 16;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+        int m, n;
+        tile_coords(t, m_tiles, n_tiles, m, n);
+        const bool ready = wait_phase(&bars->tfull[acc], acc_phase, abort);
+        if (!__all_sync(0xffffffffu, ready)) {
+            give_up(abort, flags);
+            break;
+        }
+        tc_fence_after();
+        const int row = m * kBM + quarter * 32 + lane;
+        acrl_bf16* out = logits + int64_t(row) * ldl;
+        LseAcc st = lse_empty();
+        float mx = -INFINITY;
+#pragma unroll 1
+        for (int c = 0; c < kBN / 32; ++c) {
+            uint32_t r[32];
+            __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the per-lane branches below
+            tmem_ld32(tmem + uint32_t(acc * kBN + c * 32) + lane_off, r);
+            if (c == kBN / 32 - 1) {  // the accumulator is read out: hand it back to the MMA thread
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars->tempty[acc]);
+            }
+            const int col0 = n * kBN + c * 32;
+            if (row >= M || col0 >= N) continue;
+            uint4 v[4];
+            uint32_t* w = reinterpret_cast<uint32_t*>(v);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) w[j] = pack_bf16x2(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+            if (col0 + 32 <= N) {
+                fold_vectors<4>(st, mx, v);
+                uint4* dst = reinterpret_cast<uint4*>(out + col0);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) st_stream(dst + q, v[q]);
+            } else {
+                const acrl_bf16* h = reinterpret_cast<const acrl_bf16*>(v);
+                for (int j = 0; j < N - col0; ++j) {
+                    fold_scalar(st, mx, bf16_to_float(h[j]));
+                    out[col0 + j] = h[j];
+                }
+            }
+        }
+        if (row < M) partials[int64_t(n) * M + row] = make_float4(mx, st.U, st.s0, st.s1);
+        __syncwarp();
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    lmhead_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N, int K,
+                  acrl_bf16* __restrict__ logits, int64_t ldl, float4* __restrict__ partials, int32_t* flags) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sA = base;
+    uint8_t* sB = base + kStages * kABytes;
+    Barriers* bars = reinterpret_cast<Barriers*>(base + kStages * kStageBytes);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m_tiles = (M + kBM - 1) / kBM, n_tiles = (N + kBN - 1) / kBN;
+    const int total = m_tiles * n_tiles;
+    const int k_iters = (K + kBK - 1) / kBK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&bars->full[s], 1);
+            mbar_init(&bars->empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&bars->tfull[b], 1);
+            mbar_init(&bars->tempty[b], 4);
+        }
+        mbar_init(&bars->mma_done, 1);
+        bars->abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+    }
+    if (warp == 2) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&bars->tmem_base)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = bars->tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) producer(&tmA, &tmB, sA, sB, bars, m_tiles, n_tiles, total, k_iters, flags);
+    } else if (warp == 1) {
+        if (lane == 0) mma_issuer(sA, sB, bars, tmem, total, k_iters, flags);
+    } else {
+        epilogue(bars, tmem, M, N, m_tiles, n_tiles, total, logits, ldl, partials, flags);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+    }
+}
+
+// Merge of the per-tile states of each row: lse, logp and entropy.  One
+// thread per row, tiles in order (deterministic); partials are [n_tiles][M].
+__global__ void lmhead_merge_kernel(const float4* __restrict__ partials, const acrl_bf16* __restrict__ logits, int M,
+                                    int N, int64_t ldl, int n_tiles, const int32_t* __restrict__ ids,
+                                    const uint8_t* __restrict__ mask, float* __restrict__ lse, float* __restrict__ logp,
+                                    float* __restrict__ ent, int32_t* flags) {
+    const int row = blockIdx.x * blockDim.x + threadIdx.x;
+    if (row >= M) return;
+    if (mask && mask[row] == 0) {
+        lse[row] = logp[row] = ent[row] = 0.f;
+        return;
+    }
+    LseAcc acc = lse_empty();
+    float mx = -INFINITY;
+    for (int n = 0; n < n_tiles; ++n) {
+        const float4 p = partials[int64_t(n) * M + row];
+        acc = lse_merge(acc, LseAcc{p.y, p.z, p.w});
+        mx = fmaxf(mx, p.x);
+    }
+    row_outputs(acc, mx, logits + int64_t(row) * ldl, N, ids[row], lse, logp, ent, row, flags);
+}
+
+bool encode_map(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || fn == nullptr)
+        return false;
+    auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {ld * 2};
+    const cuuint32_t box[2] = {uint32_t(kBK), box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+}  // namespace acrl
+
+using namespace acrl;
+
+extern "C" int64_t acrl_lmhead_workspace_bytes(int64_t M, int64_t N) {
+    if (M < 0 || N < 1) return -1;
+    return ((N + kBN - 1) / kBN) * M * int64_t(sizeof(float4));
+}
+
+extern "C" acrl_status acrl_lmhead_logits_stats(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t ldh,
+                                                const acrl_bf16* weight, int64_t N, int64_t ldw, acrl_bf16* logits,
+                                                int64_t ldl, float* partials, int32_t* dev_flags,
+                                                acrl_stream stream) {
+    if (M < 0 || K < 1 || N < 1 || M > kMaxGrid || N > kMaxGrid || K > kMaxGrid) return ACRL_ERR_INVALID_ARG;
+    if (ldh < K || ldw < K || ldl < N || (ldh & 7) || (ldw & 7) || (ldl & 7)) return ACRL_ERR_INVALID_ARG;
+    if (!dev_flags) return ACRL_ERR_INVALID_ARG;
+    if (M == 0) return ACRL_OK;
+    if (!hidden || !weight || !logits || !partials) return ACRL_ERR_INVALID_ARG;
+    if (!aligned16(hidden) || !aligned16(weight) || !aligned16(logits) || !aligned16(partials))
+        return ACRL_ERR_INVALID_ARG;
+    CUtensorMap tmA, tmB;
+    if (!encode_map(&tmA, hidden, uint64_t(M), uint64_t(K), uint64_t(ldh), kBM) ||
+        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN))
+        return ACRL_ERR_CUDA;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return ACRL_ERR_CUDA;
+    if (cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess)
+        return ACRL_ERR_CUDA;
+    const int64_t total = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
+    if (total > kMaxGrid) return ACRL_ERR_INVALID_ARG;
+    const int grid = int(total < sms ? total : sms);
+    lmhead_kernel<<<grid, kThreads, kSmemBytes, reinterpret_cast<cudaStream_t>(stream)>>>(
+        tmA, tmB, int(M), int(N), int(K), logits, ldl, reinterpret_cast<float4*>(partials), dev_flags);
+    return launch_status();
+}
+
+extern "C" acrl_status acrl_lmhead_merge(const float* partials, const acrl_bf16* logits, int64_t M, int64_t N,
+                                         int64_t ldl, const int32_t* ids, const uint8_t* mask, float* lse, float* logp,
+                                         float* entropy, int32_t* dev_flags, acrl_stream stream) {
+    if (M < 0 || N < 1 || N > kMaxVocab || M > kMaxGrid || ldl < N) return ACRL_ERR_INVALID_ARG;
+    if (!dev_flags) return ACRL_ERR_INVALID_ARG;
+    if (M == 0) return ACRL_OK;
+    if (!partials || !logits || !ids || !lse || !logp || !entropy) return ACRL_ERR_INVALID_ARG;
+    if (!aligned16(partials)) return ACRL_ERR_INVALID_ARG;
+    const int threads = 128;
+    lmhead_merge_kernel<<<unsigned((M + threads - 1) / threads), threads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+        reinterpret_cast<const float4*>(partials), logits, int(M), int(N), ldl, int((N + kBN - 1) / kBN), ids, mask,
+        lse, logp, entropy, dev_flags);
+    return launch_status();
+}

@@ -14,30 +14,6 @@
 namespace acrl {
 namespace {
 
-// Outputs of one row from its merged state; mx is the row maximum (natural units).
-__device__ __forceinline__ void row_outputs(const LseAcc& acc, float mx, const acrl_bf16* row, int V, int a,
-                                            float* lse, float* logp, float* ent, int64_t t, int32_t* flags) {
-    const float l2s0 = log2f(acc.s0);
-    // acc.U is mx*log2(e) rounded; c is that rounding error, exact through the FMA
-    const float c = fmaf(mx, kLog2e, -acc.U);
-    const float lse_v = fmaf(kLn2, l2s0 - c, mx);
-    const float H = kLn2 * (l2s0 - acc.s1 / acc.s0);
-    float lp = 0.f;
-    if (a >= 0 && a < V) {
-        lp = (bf16_to_float(row[a]) - mx) - kLn2 * (l2s0 - c);
-    } else {
-        raise_flag(flags, ACRL_FLAG_BAD_ID);
-    }
-    if (!isfinite(lse_v) || !isfinite(H)) {
-        raise_flag(flags, ACRL_FLAG_NONFINITE);
-        lse[t] = logp[t] = ent[t] = __int_as_float(0x7fc00000);
-        return;
-    }
-    lse[t] = lse_v;
-    logp[t] = lp;
-    ent[t] = H;
-}
-
 // A whole CTA per row (vocabulary-size rows).
 template <int THREADS, int UNROLL>
 __global__ void __launch_bounds__(THREADS) token_stats_cta(const acrl_bf16* __restrict__ logits, int64_t T, int V,

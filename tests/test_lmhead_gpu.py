@@ -1,0 +1,126 @@
+"""The fused LM-head path (tcgen05 GEMM with the log-softmax statistics in
+its epilogue, then the merge) against the float64 oracle: logits within one
+bf16 ulp of the exactly rounded product, lse/logp/entropy within the bars of
+the statistics pass, and the whole ACRL chain on the workload of 32,768
+tokens x 4,096 hidden x 151,936 vocabulary on sampled rows."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import workloads as W
+from parity import (TOL_LOGP, assert_close_abs, assert_close_rel, assert_grad_rows, assert_loss, compare_batch,
+                    compare_seq, grad_rows, host, oracle_params, rows_f64)
+
+pytestmark = pytest.mark.gpu
+
+import paper_2607_24062_gb300 as acrl  # noqa: E402
+from paper_2607_24062_gb300 import api  # noqa: E402
+
+DEV = "cuda"
+
+
+def _f64(t):
+    return t.detach().to(torch.float64).cpu().numpy()
+
+
+def _check_logits(got_bf16, ref, what="logits"):
+    """Within one bf16 ulp of the oracle's exactly rounded value."""
+    got = _f64(got_bf16)
+    ulp = np.ldexp(1.0, np.frexp(np.abs(ref))[1] - 8)
+    bad = np.abs(got - ref) > ulp * 1.0000001 + 1e-30
+    assert not bad.any(), f"{what}: {bad.sum()} of {bad.size} off by more than one bf16 ulp"
+    # and most elements identical (the GPU rounds an fp32 sum, the oracle the exact one)
+    assert np.mean(got == ref) > 0.99
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (200, 1000, 328), (384, 2304, 4096), (130, 151936, 64)])
+def test_lmhead_small_shapes(M, N, K):
+    gen = torch.Generator(device=DEV).manual_seed(M * 7 + N + K)
+    H = torch.randn((M, K), generator=gen, device=DEV).to(torch.bfloat16)
+    Wt = (0.02 * torch.randn((N, K), generator=gen, device=DEV)).to(torch.bfloat16)
+    ids = torch.randint(0, N, (M,), generator=gen, device=DEV, dtype=torch.int32)
+    mask = (torch.rand(M, generator=gen, device=DEV) < 0.9).to(torch.uint8)
+    flags = api.new_flags()
+    logits, partials = api.lmhead_logits_stats(H, Wt, N=N, flags=flags)
+    lse, logp, ent = api.lmhead_merge(partials, logits, ids, mask, N=N, flags=flags)
+    assert api.read_flags(flags) == 0
+    z = O.lmhead_logits(_f64(H), _f64(Wt))
+    _check_logits(logits[:, :N], z)
+    # merge against the statistics of the logits the GEMM stored (the epilogue's own arithmetic) ...
+    zg = rows_f64(logits, np.arange(M), N)
+    olse, ologp, oH, _ = O.token_stats(zg, host(ids), host(mask))
+    assert_close_abs(host(lse), olse, 1e-5 + 1e-6 * np.abs(olse), "lse (stored logits)")
+    assert_close_abs(host(logp), ologp, 2e-5, "logp (stored logits)")
+    assert_close_rel(host(ent), oH, rel=1e-4, floor=1e-6, what="entropy (stored logits)")
+    # ... and against the oracle's own chain
+    olse, ologp, oH, _ = O.token_stats(z, host(ids), host(mask))
+    assert_close_abs(host(lse), olse, TOL_LOGP, "lse")
+    assert_close_abs(host(logp), ologp, TOL_LOGP, "logp")
+    assert_close_rel(host(ent), oH, floor=1e-5, what="entropy")
+
+
+def test_lmhead_matches_token_stats_on_same_logits():
+    """The fused statistics equal acrl_token_stats run on the logits the GEMM wrote."""
+    M, N, K = 256, 32000, 512
+    gen = torch.Generator(device=DEV).manual_seed(5)
+    H = torch.randn((M, K), generator=gen, device=DEV).to(torch.bfloat16)
+    Wt = (0.05 * torch.randn((N, K), generator=gen, device=DEV)).to(torch.bfloat16)
+    ids = torch.randint(0, N, (M,), generator=gen, device=DEV, dtype=torch.int32)
+    logits, partials = api.lmhead_logits_stats(H, Wt, N=N)
+    lse, logp, ent = api.lmhead_merge(partials, logits, ids, None, N=N)
+    lse2, logp2, ent2 = api.token_stats(logits, ids, None, V=N)
+    torch.cuda.synchronize()
+    assert_close_abs(host(lse), host(lse2), 1e-5, "lse")
+    assert_close_abs(host(logp), host(logp2), 1e-5, "logp")
+    assert_close_rel(host(ent), host(ent2), rel=1e-5, floor=1e-6, what="entropy")
+
+
+def test_lmhead_workload_full_chain():
+    """32,768 tokens x 4,096 x 151,936: GEMM + merge, discrepancy, advantages,
+    controller, gradient on the stored logits; oracle on sampled rows."""
+    torch.cuda.empty_cache()
+    b = W.generate_lmhead(device=DEV)
+    p = acrl.Params()
+    op = oracle_params(p)
+    flags = api.new_flags()
+    logits, partials = api.lmhead_logits_stats(b.hidden, b.weight, N=b.N, flags=flags)
+    lse, logp, ent = api.lmhead_merge(partials, logits, b.ids, b.mask, N=b.N, flags=flags)
+    del partials
+    disc = api.seq_discrepancy(logp, b.logp_mu, b.mask, b.seq_offsets, b.group_offsets, ent, flags=flags)
+    adv = api.grpo_advantage(b.rewards, b.group_offsets, p, flags=flags)
+    state = api.controller_init(p)
+    w, coef, alpha = api.controller_step(state, p, disc, b.mask, b.seq_offsets, b.group_offsets, adv, flags=flags)
+    grad, tl, loss = api.loss_grad_logits(logits, b.ids, b.mask, lse, None, coef, p.clip_eps, V=b.N, flags=flags)
+    torch.cuda.synchronize()
+    assert api.read_flags(flags) == 0
+    # O(T) stages, stage-isolated on the GPU's log-probs
+    mask, so, go = host(b.mask), host(b.seq_offsets), host(b.group_offsets)
+    mu = host(b.logp_mu).astype(np.float64)
+    lr, d, seq, grp, batch, _ = O.seq_discrepancy(host(logp).astype(np.float64), mu, mask, so, go,
+                                                  host(ent).astype(np.float64))
+    compare_seq(disc.seq_host(), seq)
+    compare_batch(disc.batch_host(), batch)
+    oadv = O.grpo_advantage(host(b.rewards).astype(np.float64), go, op)
+    ow, oalpha, ost, info, _ = O.controller_step(O.controller_init(op), op, lr, mask, so, go, seq, grp, batch, oadv)
+    assert_close_rel(host(w), ow, floor=1e-7, what="weight")
+    ocoef = O.loss_coefficients(ow, oadv, mask, so, seq, grp, batch, op)
+    tl_ref, loss_ref = O.surrogate_loss(host(logp).astype(np.float64), None, oadv, ow, mask, so, seq, grp, batch, op)
+    assert_loss(float(loss), loss_ref, tl_ref)
+    # vocabulary-wide outputs on sampled rows, from the oracle's own fp64 logits
+    rng = np.random.default_rng(3)
+    rows = np.unique(np.concatenate([rng.choice(b.T, size=40, replace=False), [0, b.T - 1]]))
+    Wf = _f64(b.weight)
+    z = O.lmhead_logits(_f64(b.hidden[torch.as_tensor(rows, device=DEV)]), Wf)
+    del Wf
+    _check_logits(logits[torch.as_tensor(rows, device=DEV), :b.N], z, "logits (sampled rows)")
+    olse, ologp, oH, _ = O.token_stats(z, host(b.ids)[rows], mask[rows])
+    assert_close_abs(host(lse)[rows], olse, TOL_LOGP, "lse")
+    assert_close_abs(host(logp)[rows], ologp, TOL_LOGP, "logp")
+    assert_close_rel(host(ent)[rows], oH, floor=1e-5, what="entropy")
+    lse_full = np.zeros(b.T)
+    lse_full[rows] = olse
+    ograd, _, _ = O.loss_grad_logits(z, host(b.ids), mask, lse_full, None, oadv, ow, so, seq, grp, batch, op,
+                                     rows=rows)
+    assert_grad_rows(grad_rows(grad, rows, b.N), ograd, ocoef[rows], host(b.ids)[rows])

@@ -580,3 +580,26 @@ def test_moving_average_X_by_hand():
     assert Xs[0] == (pytest.approx(0.02), pytest.approx(0.02))
     assert Xs[1] == (pytest.approx(0.02), pytest.approx(0.03))
     assert Xs[2] == (pytest.approx(0.03), pytest.approx(0.02))
+
+
+def test_round_bf16_matches_library_and_ties():
+    rng = np.random.default_rng(12)
+    x = rng.normal(0, 3, size=20000).astype(np.float32).astype(np.float64)
+    ref = torch.tensor(x, dtype=torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(O.round_bf16(x), ref)
+    # ties go to the even mantissa: 1 + 2^-8 -> 1, 1 + 3 * 2^-8 -> 1 + 2^-6 ... (spacing 2^-7 in [1, 2))
+    assert O.round_bf16(1 + 2 ** -8) == 1.0
+    assert O.round_bf16(1 + 3 * 2 ** -8) == 1 + 2 ** -6
+    assert O.round_bf16(-(1 + 2 ** -8)) == -1.0
+    assert O.round_bf16(1 + 2 ** -8 + 2 ** -30) == 1 + 2 ** -7
+
+
+def test_lmhead_logits_small():
+    rng = np.random.default_rng(13)
+    H = O.round_bf16(rng.normal(size=(5, 40)))
+    W = O.round_bf16(rng.normal(0, 0.2, size=(7, 40)))
+    z = O.lmhead_logits(H, W)
+    for i in range(5):
+        for j in range(7):
+            exact = math.fsum(H[i, k] * W[j, k] for k in range(40))
+            assert z[i, j] == O.round_bf16(exact)

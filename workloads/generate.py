@@ -267,6 +267,80 @@ def generate(spec: WorkloadSpec, seed: int | None = None, device="cpu",
                  st.seq_offsets.to(dev), st.group_offsets.to(dev), st.T)
 
 
+# --------------------------------------------------------------------------
+# fused LM-head workload: hidden states and the LM-head weight
+# --------------------------------------------------------------------------
+
+@dataclass
+class LMHeadBatch:
+    hidden: torch.Tensor         # bf16 [T, K] ~ N(0, 1)
+    weight: torch.Tensor         # bf16 [N, K] ~ N(0, w_std^2)
+    ids: torch.Tensor            # int32 [T]
+    mask: torch.Tensor           # uint8 [T]
+    logp_mu: torch.Tensor        # float32 [T]
+    rewards: torch.Tensor        # float32 [S]
+    seq_offsets: torch.Tensor    # int64 [S+1]
+    group_offsets: torch.Tensor  # int32 [Q+1]
+    T: int
+    N: int
+    K: int
+
+    @property
+    def S(self) -> int:
+        return self.seq_offsets.numel() - 1
+
+    @property
+    def Gn(self) -> int:
+        return self.group_offsets.numel() - 1
+
+
+LMHEAD = WorkloadSpec("lmhead", 16, 8, 256, 256, 151936, dist="normal", fp8_scale="row", reward_p=0.3)
+LMHEAD_K = 4096
+LMHEAD_W_STD = 0.02
+
+
+def _rowwise_e4m3(x: torch.Tensor) -> torch.Tensor:
+    s = (x.abs().amax(dim=1, keepdim=True) / E4M3_MAX).clamp_min(1e-30)
+    return e4m3_roundtrip(x / s, "nearest") * s
+
+
+def generate_lmhead(spec: WorkloadSpec = LMHEAD, K: int = LMHEAD_K, w_std: float = LMHEAD_W_STD,
+                    seed: int | None = None, device="cpu", rows_per_chunk: int = 2048) -> LMHeadBatch:
+    """Hidden states H ~ N(0,1) and weight W ~ N(0, w_std^2) in bf16.  The
+    sampled ids come from softmax(H W^T) by Gumbel-max; mu's log-probs from the
+    rollout engine's FP8 view: H quantised per token and W per output channel
+    to E4M3 (Sec. 5.1), multiplied, log-softmax at the sampled id.  The
+    products here are torch library matmuls standing in for the two engines."""
+    if seed is None:
+        seed = seed_for("lmhead")
+    st = make_structure(spec, seed)
+    dev = torch.device(device)
+    gen = torch.Generator(device=dev).manual_seed(seed + 17)
+    T, N = st.T, spec.V
+    hidden = torch.randn((T, K), generator=gen, device=dev).to(torch.bfloat16)
+    weight = (torch.randn((N, K), generator=gen, device=dev) * w_std).to(torch.bfloat16)
+    cdt = torch.float32 if dev.type == "cpu" else torch.bfloat16
+    wq = torch.empty_like(weight)
+    for r0 in range(0, N, 8192):
+        wq[r0:r0 + 8192] = _rowwise_e4m3(weight[r0:r0 + 8192].float()).to(torch.bfloat16)
+    ids = torch.empty(T, dtype=torch.int32, device=dev)
+    logp_mu = torch.empty(T, dtype=torch.float32, device=dev)
+    for r0 in range(0, T, rows_per_chunk):
+        r1 = min(T, r0 + rows_per_chunk)
+        z = (hidden[r0:r1].to(cdt) @ weight.to(cdt).T).float()
+        u = torch.rand(z.shape, generator=gen, device=dev)
+        a = torch.argmax(z - torch.log(-torch.log(u)), dim=1)
+        del u, z
+        ids[r0:r1] = a.to(torch.int32)
+        hq = _rowwise_e4m3(hidden[r0:r1].float()).to(cdt)
+        zq = (hq @ wq.to(cdt).T).float()
+        logp_mu[r0:r1] = torch.log_softmax(zq, dim=1).gather(1, a.view(-1, 1)).view(-1)
+        del zq, hq
+    logp_mu.clamp_(max=0.0)
+    return LMHeadBatch(hidden, weight, ids, st.mask.to(dev), logp_mu, st.rewards.to(dev), st.seq_offsets.to(dev),
+                       st.group_offsets.to(dev), T, N, K)
+
+
 def small_variant(spec: WorkloadSpec, **kw) -> WorkloadSpec:
     """Same distributions at a size the oracle finishes in seconds."""
     return replace(spec, **kw)
@@ -302,7 +376,8 @@ def describe(spec: WorkloadSpec) -> str:
             f"V={spec.V} ld={spec.ld} {spec.dist}(scale={spec.scale}) fp8={spec.fp8_scale}/{spec.fp8_round}")
 
 
-__all__ = ["WorkloadSpec", "TINY", "GRPO", "QWEN", "LONG", "SPECS", "generate", "make_structure",
+__all__ = ["WorkloadSpec", "TINY", "GRPO", "QWEN", "LONG", "LMHEAD", "SPECS", "generate", "make_structure",
+           "generate_lmhead", "LMHeadBatch", "LMHEAD_K", "LMHEAD_W_STD",
            "e4m3_roundtrip", "e4m3_values", "seed_for", "small_variant", "token_level", "Batch",
            "expected_tokens", "describe", "E4M3_MAX"]
 
