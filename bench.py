@@ -359,6 +359,98 @@ def run_ours(args):
     return 0
 
 
+def _peak_tflops():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops_sustained"]), "measured (sustained)"
+    except Exception:
+        return 1700.0, "fallback (sustained)"
+
+
+def run_lmhead(args):
+    """The fused LM-head workload: 32,768 tokens x 4,096 hidden x 151,936
+    vocabulary.  A step is the GEMM with the statistics epilogue, the merge,
+    the O(T) stages and the gradient on the stored bf16 logits."""
+    import torch
+
+    import paper_2607_24062_gb300 as acrl
+    import workloads as W
+    from paper_2607_24062_gb300 import build
+
+    world, rank, local = _dist()
+    build.build()
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    spec = W.LMHEAD if args.workload == "lmhead" else W.small_variant(W.LMHEAD, name="lmhead_profile", n_prompts=2)
+    b = W.generate_lmhead(spec, device=dev)
+    p = acrl.Params()
+    M, N, K = b.T, b.N, b.K
+    stream = torch.cuda.current_stream(dev)
+    flags = acrl.api.new_flags(dev)
+    ldl = ((N + 7) // 8) * 8
+    logits = torch.empty((M, ldl), dtype=torch.bfloat16, device=dev)
+    partials = torch.empty(acrl.api.lmhead_workspace_bytes(M, N) // 4, dtype=torch.float32, device=dev)
+    f32 = dict(dtype=torch.float32, device=dev)
+    lse, logp, ent = torch.empty(M, **f32), torch.empty(M, **f32), torch.empty(M, **f32)
+    grad = torch.empty((M, ldl), dtype=torch.bfloat16, device=dev)
+    state = acrl.controller_init(p, device=dev)
+
+    def one(ev=None):
+        if ev:
+            ev[0].record(stream)
+        acrl.api.lmhead_logits_stats(b.hidden, b.weight, N=N, logits=logits, partials=partials, flags=flags)
+        if ev:
+            ev[1].record(stream)
+        acrl.api.lmhead_merge(partials, logits, b.ids, b.mask, N=N, lse=lse, logp=logp, entropy=ent, flags=flags)
+        disc = acrl.seq_discrepancy(logp, b.logp_mu, b.mask, b.seq_offsets, b.group_offsets, ent, flags=flags)
+        adv = acrl.grpo_advantage(b.rewards, b.group_offsets, p, flags=flags)
+        w, coef, alpha = acrl.controller_step(state, p, disc, b.mask, b.seq_offsets, b.group_offsets, adv,
+                                              flags=flags)
+        if ev:
+            ev[2].record(stream)
+        acrl.loss_grad_logits(logits, b.ids, b.mask, lse, None, coef, p.clip_eps, V=N, grad=grad, flags=flags)
+        if ev:
+            ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        one()
+    torch.cuda.synchronize()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index) as clocks:
+        torch.cuda.synchronize()
+        t0.record(stream)
+        for k in range(args.steps):
+            one(evs[k])
+        t1.record(stream)
+        torch.cuda.synchronize()
+    fl = acrl.read_flags(flags)
+    total_ms = t0.elapsed_time(t1)
+    gemm_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in evs]))
+    grad_ms = float(np.mean([e[2].elapsed_time(e[3]) for e in evs]))
+    flop = 2.0 * M * N * K
+    tf = flop / (gemm_ms / 1e3) / 1e12
+    peak, kind = _peak_tflops()
+    n_valid = int(b.mask.sum())
+    out = {"metric": "tokens/s fused LM-head projection + logprob + discrepancy + grad at V=151936",
+           "value": n_valid * args.steps / (total_ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "bf16 (tensor cores, fp32 accumulate)", "data": "synthetic",
+           "config": {"workload": f"lmhead: hidden bf16 [{M}, {K}] ~N(0,1), weight bf16 [{N}, {K}] ~N(0, 0.02^2), "
+                                  "mu from E4M3 per-token/per-channel copies", "flags": fl},
+           "roofline": {"bound": "tensor", "kernel": "acrl_lmhead_logits_stats", "achieved": tf, "peak": peak,
+                        "unit": "TFLOP/s", "frac": tf / peak, "traffic": None, "peak_kind": kind,
+                        "flop_per_launch": flop, "ms_per_launch": gemm_ms},
+           "kernels": {"acrl_lmhead_logits_stats": {"ms": gemm_ms, "TFLOP/s": tf},
+                       "acrl_loss_grad_logits": {"ms": grad_ms,
+                                                 "GB/s": 4.0 * M * N / (grad_ms / 1e3) / 1e9}},
+           "clocks": clocks.summary(), "gpu_launches": 11 * args.steps}
+    print(json.dumps(out))
+    return 0
+
+
 def run_e2e(batch, step, params, args, dev):
     """Same metric through the public API with the user's buffers in host
     memory: every step uploads that step's inputs from page-locked host memory,
@@ -495,6 +587,8 @@ def main():
         args.warmup = 3
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload in ("lmhead", "lmhead_profile"):
+        return run_lmhead(args)
     return run_ours(args)
 
 
