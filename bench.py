@@ -451,6 +451,20 @@ def run_lmhead(args):
     return 0
 
 
+def _huge_empty(shape, dtype):
+    """np.empty whose pages are advised as transparent huge pages (Linux), before any page is touched."""
+    import ctypes
+    arr = np.empty(shape, dtype=dtype)
+    try:
+        libc = ctypes.CDLL("libc.so.6")
+        page = os.sysconf("SC_PAGE_SIZE")
+        start = arr.ctypes.data & ~(page - 1)
+        libc.madvise(ctypes.c_void_p(start), ctypes.c_size_t(arr.nbytes + arr.ctypes.data - start), 14)
+    except Exception:
+        pass
+    return arr
+
+
 def run_e2e(batch, step, params, args, dev):
     """Same metric through the public API with the user's buffers in host
     memory: every step uploads that step's inputs from page-locked host memory,
@@ -464,9 +478,11 @@ def run_e2e(batch, step, params, args, dev):
     cudart = torch.cuda.cudart()
     T, ld = batch.logits.shape
     V = batch.V
-    # the user's host arrays, page-locked in place (torch's pinned allocator would round 44.8 GB up to 64 GB)
-    h_logits_np = np.empty((T, ld), dtype=np.uint16)
-    h_grad_np = np.empty((T, ld), dtype=np.uint16)
+    # The user's host arrays, page-locked in place (torch's pinned allocator would round 44.8 GB up to 64 GB).
+    # They are advised onto huge pages before first touch: with 64 KB pages, copies from buffers this large
+    # ran at a fraction of the link rate, with huge pages at the full rate.
+    h_logits_np = _huge_empty((T, ld), np.uint16)
+    h_grad_np = _huge_empty((T, ld), np.uint16)
     registered = []
     try:
         for arr in (h_logits_np, h_grad_np):
