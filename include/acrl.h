@@ -256,6 +256,10 @@ acrl_status acrl_controller_init(acrl_controller_state* state, const acrl_params
  * and the per-token loss coefficient of Eq. ACRL
  *     coef_t = m_t w_t A_i / norm_t,  norm_t = Q_eff G_g n_i  (or N for TOKEN_MEAN).
  * X <= 0 in ACRL mode gives alpha = 0 and raises X_NONPOS.
+ * The controller reads n_tokens, n_groups_valid and Y_sum of `batch` (and
+ * rewrites Y_mean = Y_sum / n_groups_valid): a data-parallel caller that sums
+ * those three fields over its ranks before this call gets one global X and
+ * the global loss normalisation on every rank.
  *   state     device, updated in place.
  *   lr, mask, seq_offsets, group_offsets  as for acrl_seq_discrepancy.
  *   seq       device [S] in/out (writes alpha, sum_w, n_trunc).

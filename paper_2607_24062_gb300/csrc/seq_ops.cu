@@ -237,6 +237,8 @@ __global__ void __launch_bounds__(kFinThreads) controller_alpha_kernel(
     __shared__ double sh_X;
     __shared__ int sh_apply;
     if (threadIdx.x == 0) {
+        // Y_mean from the (possibly all-reduced across ranks) sum and prompt count
+        batch->Y_mean = batch->n_groups_valid > 0 ? batch->Y_sum / double(batch->n_groups_valid) : 0.0;
         acrl_controller_state s = *st;
         const bool was_calibrated = s.calibrated != 0;
         int apply = 1;
@@ -268,7 +270,7 @@ __global__ void __launch_bounds__(kFinThreads) controller_alpha_kernel(
     __syncthreads();
     const double X = sh_X;
     const bool apply = sh_apply != 0;
-    const double Ybatch = batch->Y_mean;
+    const double Ybatch = batch->Y_mean;  // written by thread 0 above, before the barrier
     for (int i = threadIdx.x; i < S; i += kFinThreads) {
         float a = 0.f;
         const float A = adv[i];

@@ -50,13 +50,18 @@ class AcrlStep:
     def reset_controller(self, stream=None):
         api.controller_init(self.params, state=self.state, stream=stream)
 
-    def statistics(self, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, stream=None):
-        """Everything up to and including the controller (one read of the logits)."""
+    def statistics(self, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, stream=None,
+                   exchange: Callable[[torch.Tensor], None] | None = None):
+        """Everything up to and including the controller (one read of the logits).
+        `exchange`, if given, is applied to the batch-statistics bytes before the
+        controller (e.g. distributed.allreduce_batch_stats across ranks)."""
         p = self.params
         api.token_stats(logits, ids, mask, V=self.V, lse=self.lse, logp=self.logp, entropy=self.entropy,
                         flags=self.flags, stream=stream)
         api.seq_discrepancy(self.logp, logp_mu, mask, seq_offsets, group_offsets, self.entropy, out=self.disc,
                             flags=self.flags, stream=stream)
+        if exchange is not None:
+            exchange(self.disc.batch)
         api.grpo_advantage(rewards, group_offsets, p, adv=self.adv, flags=self.flags, stream=stream)
         api.controller_step(self.state, p, self.disc, mask, seq_offsets, group_offsets, self.adv,
                             weight=self.weight, coef=self.coef, alpha=self.alpha, ent_coef=self.ent_coef,
@@ -87,17 +92,19 @@ class AcrlStep:
                 on_chunk(r0, r1, g)
         api.reduce_loss(self.token_loss, loss=self.loss, stream=stream)
 
-    def run(self, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, stream=None, **grad_kw):
-        self.statistics(logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, stream=stream)
+    def run(self, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, stream=None, exchange=None,
+            **grad_kw):
+        self.statistics(logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, stream=stream,
+                        exchange=exchange)
         self.gradient(logits, ids, mask, stream=stream, **grad_kw)
 
     @classmethod
     def for_batch(cls, batch, params: Params, device="cuda", grad_rows=None):
         return cls(batch.T, batch.V, batch.ld, batch.S, batch.Gn, params, device=device, grad_rows=grad_rows)
 
-    def run_batch(self, batch, stream=None, **grad_kw):
+    def run_batch(self, batch, stream=None, exchange=None, **grad_kw):
         self.run(batch.logits, batch.ids, batch.mask, batch.logp_mu, batch.rewards, batch.seq_offsets,
-                 batch.group_offsets, stream=stream, **grad_kw)
+                 batch.group_offsets, stream=stream, exchange=exchange, **grad_kw)
 
     # host views -----------------------------------------------------------
     def seq_host(self):
