@@ -50,7 +50,9 @@ typedef enum {
     ACRL_ERR_INVALID_ARG = 1,
     ACRL_ERR_CUDA = 2,
     ACRL_ERR_NOT_IMPLEMENTED = 3,
-    ACRL_ERR_DEVICE_FLAGS = 4
+    ACRL_ERR_DEVICE_FLAGS = 4,
+    ACRL_ERR_SCRATCH_TOO_SMALL = 5  /* acrl_lmhead_stats_noalloc: the problem needs more
+                                       scratch than ACRL_LMHEAD_NOALLOC_SCRATCH_BYTES */
 } acrl_status;
 
 /* Bits of the device flags word. */
@@ -363,6 +365,34 @@ acrl_status acrl_lmhead_merge(const float* partials, const acrl_bf16* logits, in
                               int64_t ldl, const int32_t* ids, const uint8_t* mask,
                               float* lse, float* logp, float* entropy,
                               int32_t* dev_flags, acrl_stream stream);
+
+/*
+ * acrl_lmhead_stats_noalloc -- acrl_lmhead_logits_stats followed by
+ * acrl_lmhead_merge in one call that allocates nothing and takes no
+ * workspace.  The paper has no counterpart: this exists for callers that
+ * cannot allocate device memory themselves -- a plugin handed only tensors
+ * by a framework whose caching allocator already owns nearly all of HBM, or a
+ * step that must not call cudaMalloc/cudaFree (cudaFree synchronises the
+ * device).  The per-tile partial states live in one fixed device array of
+ * this library, ACRL_LMHEAD_NOALLOC_SCRATCH_BYTES (16 MiB) in size, which
+ * every GPU that loads the library holds until the process exits.
+ *   Limit: ceil(N / 256) * M * 16 bytes must fit, e.g. M <= 1765 rows at
+ *   N = 151,936 or M <= 8388 at N = 32,000; larger problems return
+ *   ACRL_ERR_SCRATCH_TOO_SMALL before anything is launched.
+ *   The first call on each device looks up the array's device address with
+ *   that device current; make that first call before any stream capture.
+ *   All calls share the array: calls that overlap on the GPU (different
+ *   streams, or different host threads, on the same device) race on it and
+ *   must be ordered by the caller.  Nothing in it needs clearing between calls.
+ *   Arguments, outputs and flags are those of the two calls it combines.
+ */
+#define ACRL_LMHEAD_NOALLOC_SCRATCH_BYTES (16LL << 20)
+acrl_status acrl_lmhead_stats_noalloc(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t ldh,
+                                      const acrl_bf16* weight, int64_t N, int64_t ldw,
+                                      acrl_bf16* logits, int64_t ldl,
+                                      const int32_t* ids, const uint8_t* mask,
+                                      float* lse, float* logp, float* entropy,
+                                      int32_t* dev_flags, acrl_stream stream);
 
 /* Copy the device flags word to *host_flags; synchronises `stream`. */
 acrl_status acrl_read_flags(const int32_t* dev_flags, int32_t* host_flags, acrl_stream stream);

@@ -19,7 +19,7 @@ HEADER = os.path.join(os.path.dirname(PKG), "include", "acrl.h")
 c_i32, c_i64, c_f32, c_f64, c_p = ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_double, ctypes.c_void_p
 
 # status codes, flag bits and enums (values fixed by include/acrl.h)
-OK, ERR_INVALID_ARG, ERR_CUDA, ERR_NOT_IMPLEMENTED, ERR_DEVICE_FLAGS = 0, 1, 2, 3, 4
+OK, ERR_INVALID_ARG, ERR_CUDA, ERR_NOT_IMPLEMENTED, ERR_DEVICE_FLAGS, ERR_SCRATCH_TOO_SMALL = 0, 1, 2, 3, 4, 5
 FLAG_BAD_ID, FLAG_NONFINITE, FLAG_BAD_OFFSETS, FLAG_X_NONPOS, FLAG_TIMEOUT = 0x1, 0x2, 0x4, 0x8, 0x10
 MODE_NONE, MODE_TIS, MODE_MIS, MODE_ACRL, MODE_ACRL_CONTINUOUS, MODE_ACRL_FALLBACK = 0, 1, 2, 3, 4, 5
 Y_GROUP, Y_SEQUENCE, Y_BATCH = 0, 1, 2
@@ -74,6 +74,8 @@ SIGNATURES = {
     "acrl_lmhead_workspace_bytes": (c_i64, [c_i64, c_i64]),
     "acrl_lmhead_logits_stats": (c_i32, [c_p, c_i64, c_i64, c_i64, c_p, c_i64, c_i64, c_p, c_i64, c_p, c_p, c_p]),
     "acrl_lmhead_merge": (c_i32, [c_p, c_p, c_i64, c_i64, c_i64, c_p, c_p, c_p, c_p, c_p, c_p, c_p]),
+    "acrl_lmhead_stats_noalloc": (c_i32, [c_p, c_i64, c_i64, c_i64, c_p, c_i64, c_i64, c_p, c_i64, c_p, c_p, c_p,
+                                          c_p, c_p, c_p, c_p]),
     "acrl_read_flags": (c_i32, [c_p, ctypes.POINTER(c_i32), c_p]),
 }
 

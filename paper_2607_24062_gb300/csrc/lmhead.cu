@@ -450,3 +450,76 @@ extern "C" acrl_status acrl_lmhead_merge(const float* partials, const acrl_bf16*
         lse, logp, entropy, dev_flags);
     return launch_status();
 }
+
+// ---------------------------------------------------------------------------
+// acrl_lmhead_stats_noalloc: the same GEMM + merge with the per-tile partial
+// states kept in a fixed device array of this library instead of a
+// caller-provided workspace, for callers that cannot allocate device memory.
+// ---------------------------------------------------------------------------
+
+#include <mutex>
+
+namespace acrl {
+namespace {
+
+constexpr int64_t kNoallocScratchBytes = ACRL_LMHEAD_NOALLOC_SCRATCH_BYTES;
+
+// Every GPU that loads this library holds this array until the process exits.
+// Its contents are whatever the last call left: the GEMM writes every entry
+// the merge then reads, so nothing needs clearing between calls.
+static __device__ __align__(256) float4 g_noalloc_partials[kNoallocScratchBytes / sizeof(float4)];
+
+constexpr int kNoallocMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+float4* g_noalloc_ptr[kNoallocMaxDevices] = {};
+
+// Device address of g_noalloc_partials on the current device, looked up once
+// per device (host code must not pass the symbol itself to a kernel).
+float4* noalloc_scratch(int dev) {
+    if (dev < 0 || dev >= kNoallocMaxDevices) return nullptr;
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (g_noalloc_ptr[dev] == nullptr) {
+        float4* ptr = nullptr;
+        if (cudaGetSymbolAddress(reinterpret_cast<void**>(&ptr), g_noalloc_partials) != cudaSuccess) return nullptr;
+        g_noalloc_ptr[dev] = ptr;
+    }
+    return g_noalloc_ptr[dev];
+}
+
+}  // namespace
+}  // namespace acrl
+
+extern "C" acrl_status acrl_lmhead_stats_noalloc(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t ldh,
+                                                 const acrl_bf16* weight, int64_t N, int64_t ldw, acrl_bf16* logits,
+                                                 int64_t ldl, const int32_t* ids, const uint8_t* mask, float* lse,
+                                                 float* logp, float* entropy, int32_t* dev_flags,
+                                                 acrl_stream stream) {
+    if (M < 0 || K < 1 || N < 1 || M > kMaxGrid || N > kMaxVocab || K > kMaxGrid) return ACRL_ERR_INVALID_ARG;
+    if (ldh < K || ldw < K || ldl < N || (ldh & 7) || (ldw & 7) || (ldl & 7)) return ACRL_ERR_INVALID_ARG;
+    if (!dev_flags) return ACRL_ERR_INVALID_ARG;
+    if (((N + kBN - 1) / kBN) * M * int64_t(sizeof(float4)) > kNoallocScratchBytes) return ACRL_ERR_SCRATCH_TOO_SMALL;
+    if (M == 0) return ACRL_OK;
+    if (!hidden || !weight || !logits || !ids || !lse || !logp || !entropy) return ACRL_ERR_INVALID_ARG;
+    if (!aligned16(hidden) || !aligned16(weight) || !aligned16(logits)) return ACRL_ERR_INVALID_ARG;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return ACRL_ERR_CUDA;
+    float4* partials = noalloc_scratch(dev);
+    if (partials == nullptr) return ACRL_ERR_CUDA;
+    CUtensorMap tmA, tmB;
+    if (!encode_map(&tmA, hidden, uint64_t(M), uint64_t(K), uint64_t(ldh), kBM) ||
+        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN))
+        return ACRL_ERR_CUDA;
+    if (cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess)
+        return ACRL_ERR_CUDA;
+    const int64_t total = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
+    const int grid = int(total < sms ? total : sms);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    lmhead_kernel<<<grid, kThreads, kSmemBytes, s>>>(tmA, tmB, int(M), int(N), int(K), logits, ldl, partials,
+                                                      dev_flags);
+    const int threads = 128;
+    lmhead_merge_kernel<<<unsigned((M + threads - 1) / threads), threads, 0, s>>>(
+        partials, logits, int(M), int(N), ldl, int((N + kBN - 1) / kBN), ids, mask, lse, logp, entropy, dev_flags);
+    return launch_status();
+}

@@ -453,6 +453,7 @@ extern "C" const char* acrl_status_string(acrl_status st) {
         case ACRL_ERR_CUDA: return "CUDA launch or runtime error";
         case ACRL_ERR_NOT_IMPLEMENTED: return "not implemented";
         case ACRL_ERR_DEVICE_FLAGS: return "device flags raised";
+        case ACRL_ERR_SCRATCH_TOO_SMALL: return "problem larger than the library's fixed scratch array";
     }
     return "unknown status";
 }
