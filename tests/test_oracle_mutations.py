@@ -1,0 +1,147 @@
+"""The pins must catch plausible mistakes in the oracle.  Each case plants one
+mistake in a copy of an oracle function (on the CPU) and runs the pins of
+that function: at least one of them must fail.  Nothing here touches the GPU
+path."""
+
+import numpy as np
+import pytest
+
+import oracle as O
+import oracle.acrl_oracle as OA
+import test_oracle_pins as P
+
+
+def _token_stats_entropy_sign(z, ids, mask):
+    lse, logp, H, f = OA._orig["token_stats"](z, ids, mask)
+    return lse, logp, -H, f
+
+
+def _token_stats_logp_index(z, ids, mask):
+    lse, logp, H, f = OA._orig["token_stats"](z, np.clip(np.asarray(ids) + 1, 0, np.asarray(z).shape[1] - 1), mask)
+    return lse, logp, H, f
+
+
+def _recompute_d_log(logp_pi, logp_mu, mask, so, go, entropy=None):
+    """Mistake: d taken on log-probabilities, |log pi - log mu|, instead of probabilities."""
+    lr, d, seq, grp, batch, f = OA._orig["seq_discrepancy"](logp_pi, logp_mu, mask, so, go, entropy)
+    d2 = np.abs(np.asarray(logp_pi, dtype=float) - np.asarray(logp_mu, dtype=float))
+    m = np.ones(len(d2), dtype=bool) if mask is None else np.asarray(mask) != 0
+    d2 = np.where(m, d2, 0.0)
+    so = np.asarray(so)
+    for i in range(len(so) - 1):
+        sl = slice(so[i], so[i + 1])
+        if seq["n"][i]:
+            seq["mean_d"][i] = d2[sl][m[sl]].sum() / seq["n"][i]
+    for g in range(len(go) - 1):
+        members = [i for i in range(go[g], go[g + 1]) if seq["n"][i] > 0]
+        grp["Y"][g] = sum(seq["mean_d"][i] for i in members) / len(members) if members else 0.0
+    return lr, d2, seq, grp, batch, f
+
+
+def _grpo_ddof_ignored(rewards, group_offsets, params):
+    p = O.Params(**{**vars(params), "adv_ddof": 0})
+    return OA._orig["grpo_advantage"](rewards, group_offsets, p)
+
+
+def _grpo_no_centering(rewards, group_offsets, params):
+    A = OA._orig["grpo_advantage"](rewards, group_offsets, params)
+    return A + 0.1
+
+
+def _controller_alpha_sign(state, params, *args):
+    p = O.Params(**{**vars(params), "gamma": -params.gamma})
+    return OA._orig["controller_step"](state, p, *args)
+
+
+def _controller_no_truncation(state, params, *args):
+    p = O.Params(**{**vars(params), "C": 1e30})
+    return OA._orig["controller_step"](state, p, *args)
+
+
+def _loss_grad_sign(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch, params, rows=None):
+    """Mistake: gradient of J instead of L = -J (sign flipped)."""
+    grad, tl, loss = OA._orig["loss_grad_logits"](z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp,
+                                                  batch, params, rows)
+    return -grad, tl, loss
+
+
+def _loss_grad_wrong_column(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch, params,
+                            rows=None):
+    """Mistake: the one-hot subtracted at the neighbouring column."""
+    V = np.asarray(z).shape[1]
+    shifted = (np.asarray(ids) + 1) % V
+    grad, tl, loss = OA._orig["loss_grad_logits"](z, shifted, mask, lse, old_logp, adv, weight, seq_offsets, seq,
+                                                  grp, batch, params, rows)
+    return grad, tl, loss
+
+
+def _loss_grad_no_norm(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch, params, rows=None):
+    b2 = dict(batch)
+    b2["n_groups_valid"] = 1
+    return OA._orig["loss_grad_logits"](z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, b2, params,
+                                        rows)
+
+
+def _round_bf16_truncates(x):
+    x = np.asarray(x, dtype=np.float64)
+    f, e = np.frexp(x)
+    return np.ldexp(np.trunc(f * 256.0) / 256.0, e)
+
+
+PIN_GROUPS = {
+    "token_stats": [lambda: P.test_token_stats_matches_bruteforce(7), P.test_token_stats_library_routines,
+                    P.test_two_way_closed_form],
+    "seq_discrepancy": [P.test_distance_is_on_probabilities, P.test_hand_worked_aggregates,
+                        P.test_aggregates_as_linear_functional],
+    "grpo_advantage": [lambda: P.test_grpo_binary_closed_form(8, 3), P.test_grpo_matches_scipy_zscore,
+                       P.test_grpo_special_groups],
+    "controller_step": [lambda: [P.test_quadrant_sign_table(r) for r in P._read_quadrants()],
+                        P.test_controller_special_cases, P.test_tis_and_mis_thresholds],
+    "loss_grad_logits": [lambda: P.test_gradient_matches_autograd(False, 0.0), P.test_on_policy_loss_by_hand_and_invariants,
+                         lambda: P.test_gradient_central_differences(0.0)],
+    "round_bf16": [P.test_round_bf16_matches_library_and_ties],
+}
+
+MUTATIONS = [
+    ("token_stats", "entropy sign flipped", _token_stats_entropy_sign),
+    ("token_stats", "log-prob of the wrong column", _token_stats_logp_index),
+    ("seq_discrepancy", "distance on log-probabilities", _recompute_d_log),
+    ("grpo_advantage", "std with ddof 0 instead of 1", _grpo_ddof_ignored),
+    ("grpo_advantage", "advantage not centred", _grpo_no_centering),
+    ("controller_step", "alpha with the wrong sign", _controller_alpha_sign),
+    ("controller_step", "weights never truncated at C", _controller_no_truncation),
+    ("loss_grad_logits", "gradient sign flipped", _loss_grad_sign),
+    ("loss_grad_logits", "one-hot at the wrong column", _loss_grad_wrong_column),
+    ("loss_grad_logits", "prompt count left out of the normalisation", _loss_grad_no_norm),
+    ("round_bf16", "truncation instead of round-to-nearest-even", _round_bf16_truncates),
+]
+
+
+@pytest.fixture
+def mutate(monkeypatch):
+    if not hasattr(OA, "_orig"):
+        OA._orig = {name: getattr(OA, name) for name in PIN_GROUPS}
+
+    def apply(name, fn):
+        monkeypatch.setattr(OA, name, fn)
+        monkeypatch.setattr(O, name, fn)
+        monkeypatch.setattr(P.O, name, fn)
+    return apply
+
+
+@pytest.mark.parametrize("target,what,fn", MUTATIONS, ids=[m[1] for m in MUTATIONS])
+def test_pins_catch_planted_mistake(mutate, target, what, fn):
+    mutate(target, fn)
+    caught = 0
+    for pin in PIN_GROUPS[target]:
+        try:
+            pin()
+        except AssertionError:
+            caught += 1
+    assert caught > 0, f"no pin caught: {what}"
+
+
+def test_unmutated_oracle_passes_the_same_pins():
+    for pins in PIN_GROUPS.values():
+        for pin in pins:
+            pin()
