@@ -310,6 +310,17 @@ def run_ours(args):
         tokens_all = float(nt)
     else:
         tokens_all = float(n_valid)
+    # cached-old variant: the gradient call recomputes each row's LSE itself (a second sweep over the row);
+    # the weights would come from cached old log-probs, here the statistics pass's own
+    n_co = min(5, args.steps)
+    co_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_co)]
+    for k in range(n_co):
+        co_ev[k][0].record(stream)
+        acrl.loss_grad_logits(batch.logits, batch.ids, batch.mask, None, step.logp, step.coef, params.clip_eps,
+                              V=V, grad=step.grad, token_loss=step.token_loss, loss=step.loss, flags=step.flags)
+        co_ev[k][1].record(stream)
+    torch.cuda.synchronize()
+    co_ms = float(np.mean([a.elapsed_time(b) for a, b in co_ev]))
     k1_ms = [ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps)]
     mid_ms = [ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps)]
     k5_ms = [ev[k][2].elapsed_time(ev[k][3]) for k in range(args.steps)]
@@ -349,6 +360,9 @@ def run_ours(args):
                                  "traffic": traffic_of("token_stats.cu")},
             "acrl_loss_grad_logits": {"ms": k5_avg, "GB/s": k5_gbs, "frac": k5_gbs / peak, "bytes": k5_bytes},
             "seq_discrepancy+grpo_advantage+controller_step": {"ms": float(np.mean(mid_ms))},
+            "acrl_loss_grad_logits (lse recomputed, cached-old)": {
+                "ms": co_ms, "GB/s": k5_bytes / (co_ms / 1e3) / 1e9, "frac": k5_bytes / (co_ms / 1e3) / 1e9 / peak,
+                "note": "algorithmic bytes as the streaming call (the recompute sweep's re-read is not counted)"},
             "whole_step_GB/s": (k1_bytes + k5_bytes) / (ms_per_step / 1e3) / 1e9,
         },
         "clocks": clocks.summary(),

@@ -74,17 +74,20 @@ __device__ __forceinline__ uint4 grad_vec(const uint4 v, const RowPlan& rp, int 
     return o;
 }
 
-template <int TEAM, int UNROLL, bool ENT>
+// LAST: this is the second sweep over a row whose lines the first sweep kept in
+// L2, and the last read of them (L2 evict-first policy).
+template <int TEAM, int UNROLL, bool ENT, bool LAST = false>
 __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ row, acrl_bf16* __restrict__ grow, int V,
                                                 int tid, const RowPlan& rp) {
     const int nvec = V >> 3;
     const uint4* src = reinterpret_cast<const uint4*>(row);
     uint4* dst = reinterpret_cast<uint4*>(grow);
+    const uint64_t pol = LAST ? policy_evict_first() : 0;
     int v = tid;
     for (; v + (UNROLL - 1) * TEAM < nvec; v += UNROLL * TEAM) {
         uint4 buf[UNROLL];
 #pragma unroll
-        for (int k = 0; k < UNROLL; ++k) buf[k] = ld_stream(src + v + k * TEAM);
+        for (int k = 0; k < UNROLL; ++k) buf[k] = LAST ? ld_policy(src + v + k * TEAM, pol) : ld_stream(src + v + k * TEAM);
 #pragma unroll
         for (int k = 0; k < UNROLL; ++k) {
             const int vi = v + k * TEAM;
@@ -169,7 +172,7 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
     if (live) {
         if (RECOMPUTE) {
             float mx;
-            LseAcc acc = warp_lse(row_partial<TEAM, UNROLL>(row, V, tid, mx));
+            LseAcc acc = warp_lse(row_partial<TEAM, UNROLL, true>(row, V, tid, mx));
             if (TEAM > 32) {
                 constexpr int NW = TEAM / 32;
                 if ((tid & 31) == 0) part[tid >> 5] = acc;
@@ -197,7 +200,7 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
     if (c == 0.f && e == 0.f) {
         zero_row<TEAM>(grow, V, tid);
     } else {
-        stream_grad_row<TEAM, UNROLL, ENT>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a));
+        stream_grad_row<TEAM, UNROLL, ENT, RECOMPUTE>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a));
     }
 }
 

@@ -97,7 +97,9 @@ extern "C" acrl_status acrl_token_stats(const acrl_bf16* logits, int64_t T, int6
         token_stats_warp<THREADS, 4><<<unsigned(grid_for(THREADS / 32, T)), THREADS, 0, s>>>(
             logits, T, v, ld, ids, mask, lse, logp, entropy, dev_flags);
     } else {
-        constexpr int THREADS = 512;
+        // 128 threads per row: many independent rows in flight per SM and a short
+        // end-of-row merge (measured best of 128/256/512/1024 and a warp per row)
+        constexpr int THREADS = 128;
         token_stats_cta<THREADS, 4><<<unsigned(grid_for(1, T)), THREADS, 0, s>>>(
             logits, T, v, ld, ids, mask, lse, logp, entropy, dev_flags);
     }
