@@ -40,12 +40,12 @@ FALLBACK_HBM_GBS = 6800.0
 LAUNCHES_PER_STEP = 9
 # DRAM traffic of one gradient-kernel launch on the bench workload, from ncu
 # (dram__bytes_read.sum + dram__bytes_write.sum), valid only for the kernel source
-# it was taken on (sha256 of the file, first 16 hex digits).
+# it was taken on (sha256 of the file and the device headers, first 16 hex digits).
 # Taken with `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` (one pass) on the
 # bench workload; see profiles/dram_traffic_qwen_bench.md.
 NCU_TRAFFIC = {
-    "loss_grad.cu": {"src": "0a208a2210e7f12c", "bytes_per_launch": 41.71e9 + 44.87e9},
-    "token_stats.cu": {"src": "4c54a894cb214469", "bytes_per_launch": 44.93e9 + 3.45e6},
+    "loss_grad.cu": {"src": "2c11cdde91747dde", "bytes_per_launch": 41.71e9 + 44.87e9},
+    "token_stats.cu": {"src": "00adc393084e33b9", "bytes_per_launch": 44.94e9 + 3.74e6},
 }
 
 
@@ -60,9 +60,12 @@ def _peaks():
 
 
 def _src_hash(name):
-    p = os.path.join(ROOT, "paper_2607_24062_gb300", "csrc", name)
-    with open(p, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    """Hash of a kernel source and the device headers it includes."""
+    d = hashlib.sha256()
+    for f in (name, "acrl_device.cuh", "row_lse.cuh", "acrl_host.h"):
+        with open(os.path.join(ROOT, "paper_2607_24062_gb300", "csrc", f), "rb") as fh:
+            d.update(fh.read())
+    return d.hexdigest()[:16]
 
 
 class ClockSampler:
