@@ -150,15 +150,26 @@ __device__ __forceinline__ RowPlan make_plan(float c, float e, float L, float H,
     return rp;
 }
 
-// One row handled by a team (a whole CTA, or one warp).  `part` is the CTA's
-// shared scratch for the recompute sweep (unused by warp teams).
+// lse and logp = z_a - lse of a row from its merged state and maximum, in the
+// same form as the statistics kernel (the rounding of max*log2(e) corrected
+// exactly through an FMA).
+__device__ __forceinline__ void lse_logp(const LseAcc& acc, float mx, float za, float& L, float& lp) {
+    const float l2s0 = log2f(acc.s0);
+    const float c = fmaf(mx, kLog2e, -acc.U);
+    L = fmaf(kLn2, l2s0 - c, mx);
+    lp = (za - mx) - kLn2 * (l2s0 - c);
+}
+
+// One row handled by a team (a whole CTA, or one warp).  `part`/`part_mx` are
+// the CTA's shared scratch for the recompute sweep (unused by warp teams).
 template <int TEAM, int UNROLL, bool RECOMPUTE, bool ENT>
 __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, int64_t t, int V, int64_t ld,
                                          const int32_t* __restrict__ ids, const uint8_t* __restrict__ mask,
                                          const float* __restrict__ lse, const float* __restrict__ old_logp,
                                          const float* __restrict__ coef, const float* __restrict__ entropy,
                                          const float* __restrict__ ent_coef, float eps, acrl_bf16* __restrict__ grad,
-                                         float* __restrict__ token_loss, int32_t* flags, int tid, LseAcc* part) {
+                                         float* __restrict__ token_loss, int32_t* flags, int tid, LseAcc* part,
+                                         float* part_mx) {
     const acrl_bf16* row = logits + t * ld;
     acrl_bf16* grow = grad + t * ld;
     const bool m = mask ? mask[t] != 0 : true;
@@ -170,24 +181,32 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
     const bool live = m && !bad_id && (c0 != 0.f || e != 0.f);
     float c = 0.f, loss = 0.f, L = 0.f, H = 0.f, za = 0.f, lp = 0.f;
     if (live) {
+        za = bf16_to_float(row[a]);
         if (RECOMPUTE) {
             float mx;
             LseAcc acc = warp_lse(row_partial<TEAM, UNROLL, true>(row, V, tid, mx));
+            mx = warp_max(mx);
             if (TEAM > 32) {
                 constexpr int NW = TEAM / 32;
-                if ((tid & 31) == 0) part[tid >> 5] = acc;
+                if ((tid & 31) == 0) {
+                    part[tid >> 5] = acc;
+                    part_mx[tid >> 5] = mx;
+                }
                 __syncthreads();
                 acc = part[0];
+                mx = part_mx[0];
 #pragma unroll
-                for (int w = 1; w < NW; ++w) acc = lse_merge(acc, part[w]);
+                for (int w = 1; w < NW; ++w) {
+                    acc = lse_merge(acc, part[w]);
+                    mx = fmaxf(mx, part_mx[w]);
+                }
                 __syncthreads();
             }
-            L = kLn2 * (acc.U + log2f(acc.s0));
+            lse_logp(acc, mx, za, L, lp);
         } else {
             L = lse[t];
+            lp = za - L;
         }
-        za = bf16_to_float(row[a]);
-        lp = za - L;
         const RowCoef rc = row_coef(c0, lp, old_logp, t, eps);
         c = rc.c;
         loss = rc.loss;
@@ -211,9 +230,10 @@ __global__ void __launch_bounds__(THREADS) loss_grad_cta(
     const float* __restrict__ coef, const float* __restrict__ entropy, const float* __restrict__ ent_coef, float eps,
     acrl_bf16* __restrict__ grad, float* __restrict__ token_loss, int32_t* flags) {
     __shared__ LseAcc part[THREADS / 32];
+    __shared__ float part_mx[THREADS / 32];
     for (int64_t t = blockIdx.x; t < T; t += gridDim.x)
         grad_row<THREADS, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
-                                                  eps, grad, token_loss, flags, threadIdx.x, part);
+                                                  eps, grad, token_loss, flags, threadIdx.x, part, part_mx);
 }
 
 template <int THREADS, int UNROLL, bool RECOMPUTE, bool ENT>
@@ -226,7 +246,7 @@ __global__ void __launch_bounds__(THREADS) loss_grad_warp(
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     for (int64_t t = int64_t(blockIdx.x) * NW + wid; t < T; t += int64_t(gridDim.x) * NW)
         grad_row<32, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps,
-                                             grad, token_loss, flags, lane, nullptr);
+                                             grad, token_loss, flags, lane, nullptr, nullptr);
 }
 
 // Scalar loss: sum of token losses in a fixed order.  Each thread adds float4

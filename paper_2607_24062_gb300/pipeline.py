@@ -106,6 +106,21 @@ class AcrlStep:
         self.run(batch.logits, batch.ids, batch.mask, batch.logp_mu, batch.rewards, batch.seq_offsets,
                  batch.group_offsets, stream=stream, exchange=exchange, **grad_kw)
 
+    def capture(self, batch, exchange=None, **grad_kw):
+        """Record one whole step over `batch`'s buffers as a CUDA graph (the
+        kernels' launches only; no host work is left in the step).  Returns the
+        torch.cuda.CUDAGraph; `graph.replay()` runs the step again on whatever
+        the buffers then hold.  `exchange` must be capturable (e.g. NCCL)."""
+        side = torch.cuda.Stream(device=self.lse.device)
+        side.wait_stream(torch.cuda.current_stream(self.lse.device))
+        with torch.cuda.stream(side):           # one eager run on the capture stream first
+            self.run_batch(batch, exchange=exchange, **grad_kw)
+        torch.cuda.current_stream(self.lse.device).wait_stream(side)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            self.run_batch(batch, exchange=exchange, **grad_kw)
+        return graph
+
     # host views -----------------------------------------------------------
     def seq_host(self):
         return self.disc.seq_host()

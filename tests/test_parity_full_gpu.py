@@ -118,6 +118,17 @@ def test_full_size_workload(name):
     rows, whole = _sample_rows(b, rng)
     _check_rows(step, b, rows, ref, op)
     _oracle_chain_on_whole(step, b, whole, op)
+    # cached-old path (lse recomputed inside the gradient call; at V = 151,936 a cluster of CTAs keeps each row
+    # in shared memory) on the first 4,096 rows: the same gradient as the streaming call
+    R = min(4096, b.T)
+    g2, tl2, _ = api.loss_grad_logits(b.logits[:R], b.ids[:R], b.mask[:R], None, step.logp[:R], step.coef[:R],
+                                      p.clip_eps, V=b.V)
+    torch.cuda.synchronize()
+    rr = np.arange(0, R, 7)
+    ref = grad_rows(step.grad, rr, b.V)
+    assert_grad_rows(grad_rows(g2, rr, b.V), ref, np.abs(host(step.coef)[rr]) + 1e-30, host(b.ids)[rr],
+                     what="grad (lse recomputed)")
+    assert_close_rel(host(tl2), host(step.token_loss)[:R], rel=1e-4, floor=1e-12, what="token_loss (lse recomputed)")
     # masked rows: zero gradient and zero statistics
     masked = np.flatnonzero(host(b.mask) == 0)
     if len(masked):

@@ -381,3 +381,21 @@ def test_controller_trajectory_50_steps():
         assert_close_rel(host(alpha), oalpha, floor=1e-6, what=f"alpha step {k}")
         Xs.append(float(st["X"]))
     assert all(x == Xs[0] for x in Xs)     # frozen after step 0, bit for bit
+
+
+def test_cuda_graph_replay_matches_eager():
+    """The step captured as a CUDA graph and replayed gives the eager step's outputs bit for bit."""
+    spec = W.small_variant(W.GRPO, name="graph", n_prompts=2, group_size=4, len_lo=20, len_hi=200, V=32000)
+    b = _gen(spec, seed=12)
+    p = acrl.Params(X_init=0.013)     # a fixed X: every replay is the same computation
+    eager = acrl.AcrlStep.for_batch(b, p)
+    eager.run_batch(b)
+    captured = acrl.AcrlStep.for_batch(b, p)
+    graph = captured.capture(b)
+    captured.grad.zero_()
+    graph.replay()
+    torch.cuda.synchronize()
+    for x, y in ((eager.lse, captured.lse), (eager.weight, captured.weight), (eager.coef, captured.coef),
+                 (eager.loss, captured.loss), (eager.grad, captured.grad)):
+        assert torch.equal(x.view(torch.int16) if x.dtype == torch.bfloat16 else x,
+                           y.view(torch.int16) if y.dtype == torch.bfloat16 else y)
