@@ -152,6 +152,22 @@ def read_state(state: torch.Tensor) -> np.void:
     return read_structs(state, STATE_DTYPE, 1)[0]
 
 
+def save_state(state: torch.Tensor) -> bytes:
+    """The controller state's 48 bytes, for a checkpoint (the state is plain data)."""
+    return bytes(state[: STATE_DTYPE.itemsize].cpu().numpy().tobytes())
+
+
+def load_state(blob: bytes, state: torch.Tensor | None = None, device=None) -> torch.Tensor:
+    """Restore a controller state saved by save_state; resuming from it is bit-exact."""
+    if len(blob) != STATE_DTYPE.itemsize:
+        raise AcrlError("controller state: wrong size")
+    host = torch.frombuffer(bytearray(blob), dtype=torch.uint8)
+    if state is None:
+        state = struct_buffer(STATE_DTYPE, 1, device)
+    state[: STATE_DTYPE.itemsize].copy_(host)
+    return state
+
+
 def controller_step(state, params: Params, disc: Discrepancy, mask, seq_offsets, group_offsets, adv, *, weight=None,
                     coef=None, alpha=None, ent_coef=None, flags=None, stream=None):
     """acrl_controller_step.  Returns (weight [T], coef [T], alpha [S]); the
@@ -270,5 +286,5 @@ def read_flags(flags, stream=None) -> int:
 
 __all__ = ["Params", "AcrlError", "token_stats", "seq_discrepancy", "grpo_advantage", "controller_init",
            "controller_step", "loss_grad_logits", "reduce_loss", "read_flags", "read_state", "Discrepancy",
-           "lmhead_logits_stats", "lmhead_merge", "lmhead_workspace_bytes",
+           "lmhead_logits_stats", "lmhead_merge", "lmhead_workspace_bytes", "save_state", "load_state",
            "struct_buffer", "read_structs", "new_flags", "_abi"]
