@@ -394,6 +394,15 @@ acrl_status acrl_lmhead_stats_noalloc(const acrl_bf16* hidden, int64_t M, int64_
                                       float* lse, float* logp, float* entropy,
                                       int32_t* dev_flags, acrl_stream stream);
 
+/*
+ * acrl_selftest_wait_timeout -- failure-detection self-test: one warp waits on
+ * a shared-memory barrier that nothing arrives on, with the same bounded wait
+ * that guards every pipeline wait of acrl_lmhead_logits_stats; after
+ * `limit_ns` (at most 2e9) it raises ACRL_FLAG_TIMEOUT in *dev_flags and
+ * returns, leaving the context usable.  Not part of the paper's method.
+ */
+acrl_status acrl_selftest_wait_timeout(int32_t* dev_flags, int64_t limit_ns, acrl_stream stream);
+
 /* Copy the device flags word to *host_flags; synchronises `stream`. */
 acrl_status acrl_read_flags(const int32_t* dev_flags, int32_t* host_flags, acrl_stream stream);
 

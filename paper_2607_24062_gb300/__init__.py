@@ -8,6 +8,7 @@ library; the first call does, and fails loudly if it has not been built.
 """
 
 from ._abi import (AGG_SEQ_MEAN_TOKEN_MEAN, AGG_TOKEN_MEAN, FLAG_BAD_ID, FLAG_BAD_OFFSETS, FLAG_NONFINITE,  # noqa: F401
+                   FLAG_TIMEOUT,
                    FLAG_X_NONPOS, MODE_ACRL, MODE_ACRL_CONTINUOUS, MODE_ACRL_FALLBACK, MODE_MIS, MODE_NONE,
                    MODE_TIS, SINGLETON_MEAN0_STD1, SINGLETON_ZERO, Y_BATCH, Y_GROUP, Y_SEQUENCE, AcrlError, Params)
 from .api import (controller_init, controller_step, grpo_advantage, loss_grad_logits, read_flags,  # noqa: F401

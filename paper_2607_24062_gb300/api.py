@@ -14,7 +14,7 @@ import numpy as np
 import torch
 
 from . import _abi
-from ._abi import BATCH_DTYPE, GRP_DTYPE, SEQ_DTYPE, STATE_DTYPE, AcrlError, Params, check, lib
+from ._abi import BATCH_DTYPE, GRP_DTYPE, SEQ_DTYPE, STATE_DTYPE, AcrlError, Params, check, lib  # noqa: F401
 
 
 def _ptr(t: torch.Tensor | None) -> int | None:

@@ -24,6 +24,7 @@
 #include "acrl_device.cuh"
 #include "acrl_host.h"
 #include "row_lse.cuh"
+#include "mbarrier.cuh"
 
 namespace acrl {
 namespace {
@@ -35,7 +36,6 @@ constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
 constexpr int kBandM = 16;
-constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s: every legitimate wait is microseconds
 // Instruction descriptor of tcgen05.mma kind::f16: D f32 (bits 4-5 = 1),
 // A and B bf16 (bits 7-9, 10-12 = 1), both K-major, N/8 at bit 17, M/16 at bit 24.
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kBN >> 3) << 17) |
@@ -56,54 +56,6 @@ constexpr int kSmemBytes = 1024 + kStages * kStageBytes + int(sizeof(Barriers));
 // ---------------------------------------------------------------------------
 // PTX wrappers
 // ---------------------------------------------------------------------------
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-__device__ __forceinline__ uint64_t global_ns() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-// Wait for the completion of the phase of `bar` with parity `parity`.  Gives
-// up after kWaitNs, or early once another role has set *abort (unless abort
-// is null).
-__device__ __noinline__ bool wait_phase(uint64_t* bar, uint32_t parity, volatile int32_t* abort) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = global_ns();
-    for (uint32_t i = 1;; ++i) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 255u) == 0u) {
-            if (abort && *abort) return false;
-            if (global_ns() - t0 > kWaitNs) return false;
-        }
-    }
-}
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
     asm volatile(

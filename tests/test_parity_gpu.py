@@ -424,3 +424,19 @@ def test_checkpoint_resume_is_bit_exact():
     resumed = run(api.load_state(blob), 3, 6)
     for (w1, s1), (w2, s2) in zip(full[3:], resumed):
         assert torch.equal(w1, w2) and s1 == s2
+
+
+def test_bounded_wait_reports_timeout_and_context_survives():
+    """A pipeline wait on a barrier nothing arrives on gives up after its limit and reports
+    ACRL_FLAG_TIMEOUT; the context keeps working afterwards."""
+    import time
+    flags = api.new_flags()
+    t0 = time.perf_counter()
+    api.check(api.lib().acrl_selftest_wait_timeout(flags.data_ptr(), 50_000_000,
+                                                   torch.cuda.current_stream().cuda_stream), "selftest")
+    assert api.read_flags(flags) == acrl.FLAG_TIMEOUT
+    assert time.perf_counter() - t0 < 30.0
+    logits, ids = _tiny_manual(8, 64)
+    lse, logp, H = api.token_stats(logits, ids, None, V=64)      # the context still runs kernels
+    torch.cuda.synchronize()
+    assert torch.all(torch.isfinite(lse))
