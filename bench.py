@@ -341,18 +341,21 @@ def run_ours(args):
     traffic = traffic_of("loss_grad.cu")
 
     # the same step replayed from a CUDA graph (launch gaps removed); reported beside the eager step
-    graph = step.capture(batch, exchange=exchange)
-    for _ in range(3):
-        graph.replay()
-    torch.cuda.synchronize()
-    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    g0.record(stream)
-    for _ in range(args.steps):
-        graph.replay()
-    g1.record(stream)
-    torch.cuda.synchronize()
-    graph_ms = g0.elapsed_time(g1) / args.steps
-    del graph
+    # (single process only: the multi-rank step keeps its collective outside any graph)
+    graph_ms = None
+    if world == 1:
+        graph = step.capture(batch)
+        for _ in range(3):
+            graph.replay()
+        torch.cuda.synchronize()
+        g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        for _ in range(args.steps):
+            graph.replay()
+        g1.record(stream)
+        torch.cuda.synchronize()
+        graph_ms = g0.elapsed_time(g1) / args.steps
+        del graph
 
     e2e = None
     if not args.no_e2e and rank == 0:
@@ -381,7 +384,8 @@ def run_ours(args):
                 "ms": co_ms, "GB/s": k5_bytes / (co_ms / 1e3) / 1e9, "frac": k5_bytes / (co_ms / 1e3) / 1e9 / peak,
                 "note": "algorithmic bytes as the streaming call (the recompute sweep's re-read is not counted)"},
             "whole_step_GB/s": (k1_bytes + k5_bytes) / (ms_per_step / 1e3) / 1e9,
-            "step_replayed_from_cuda_graph": {"ms": graph_ms, "tokens/s": n_valid / (graph_ms / 1e3)},
+            "step_replayed_from_cuda_graph": ({"ms": graph_ms, "tokens/s": n_valid / (graph_ms / 1e3)}
+                                              if graph_ms else None),
         },
         "clocks": clocks.summary(),
         "gpu_launches": LAUNCHES_PER_STEP * args.steps,
