@@ -440,3 +440,35 @@ def test_bounded_wait_reports_timeout_and_context_survives():
     lse, logp, H = api.token_stats(logits, ids, None, V=64)      # the context still runs kernels
     torch.cuda.synchronize()
     assert torch.all(torch.isfinite(lse))
+
+
+def test_empty_batch_through_every_call():
+    """T = 0, no responses, no prompts: every call accepts it and the outputs are zeros."""
+    p = acrl.Params()
+    step = acrl.AcrlStep(0, 64, 64, 0, 0, p)
+    z = torch.zeros((0, 64), dtype=torch.bfloat16, device=DEV)
+    e32 = torch.zeros(0, dtype=torch.int32, device=DEV)
+    step.run(z, e32, torch.zeros(0, dtype=torch.uint8, device=DEV), torch.zeros(0, device=DEV),
+             torch.zeros(0, device=DEV), torch.zeros(1, dtype=torch.int64, device=DEV),
+             torch.zeros(1, dtype=torch.int32, device=DEV))
+    torch.cuda.synchronize()
+    b = step.batch_host()
+    assert int(b["n_tokens"]) == 0 and int(b["n_groups_valid"]) == 0 and float(step.loss) == 0.0
+    assert api.read_flags(step.flags) == acrl.FLAG_X_NONPOS     # nothing to calibrate X on
+
+
+def test_fully_masked_batch():
+    """Every token masked: zero statistics, weights, coefficients, gradient and loss; X cannot be calibrated."""
+    spec = W.small_variant(W.GRPO, name="allmasked", n_prompts=2, group_size=3, len_lo=10, len_hi=40, V=3000)
+
+    def mutate(b):
+        b.mask.zero_()
+    b = _gen(spec, seed=2, mutate=mutate)
+    step = acrl.AcrlStep.for_batch(b, acrl.Params())
+    step.grad.fill_(1.0)
+    step.run_batch(b)
+    torch.cuda.synchronize()
+    assert torch.all(step.logp == 0) and torch.all(step.weight == 0) and torch.all(step.coef == 0)
+    assert torch.all(step.grad[:, :b.V] == 0) and float(step.loss) == 0.0
+    assert int(step.batch_host()["n_tokens"]) == 0
+    assert api.read_flags(step.flags) == acrl.FLAG_X_NONPOS
