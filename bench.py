@@ -542,10 +542,9 @@ def run_e2e(batch, step, params, args, dev):
         loss_h = torch.empty(1, dtype=torch.float32, pin_memory=True)
         d_logits = batch.logits
         comp = torch.cuda.current_stream(dev)
-        # Both directions share one copy stream: on this link a download running at the same time as an
-        # upload slowed the pair to a fraction of either alone, so the copies are kept one-way at a time
-        # while the kernels overlap them.
-        s_in = s_out = torch.cuda.Stream(dev)
+        # One copy stream per direction: the next step's uploads run while this step's gradient downloads,
+        # which moves more bytes per second over the host link than either direction alone.
+        s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
         nchunk = max(1, args.e2e_chunks)
         bounds = [(T * k // nchunk, T * (k + 1) // nchunk) for k in range(nchunk)]
         E = torch.cuda.Event
@@ -635,7 +634,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="qwen")
-    ap.add_argument("--e2e-steps", type=int, default=4)
+    ap.add_argument("--e2e-steps", type=int, default=8)
     ap.add_argument("--e2e-chunks", type=int, default=16)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
