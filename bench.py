@@ -33,6 +33,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "tokens/s fused logprob+discrepancy+grad at V=151936; HBM GB/s vs peak"
+LMHEAD_METRIC = "tokens/s fused LM-head projection + logprob + discrepancy + grad at V=151936"
 UNIT = "tokens/s"
 FALLBACK_HBM_GBS = 6800.0
 # Kernel launches per step inside the timed region: token_stats 1, seq_discrepancy 2,
@@ -137,6 +138,15 @@ def _dist():
     return world, rank, local
 
 
+def _lmhead_spec(W, name):
+    return W.LMHEAD if name == "lmhead" else W.small_variant(W.LMHEAD, name="lmhead_profile", n_prompts=2)
+
+
+def _lmhead_desc(b):
+    return (f"lmhead: hidden bf16 [{b.T}, {b.K}] ~N(0,1), weight bf16 [{b.N}, {b.K}] ~N(0, 0.02^2), "
+            "mu from E4M3 per-token/per-channel copies")
+
+
 def _workload_desc(spec):
     return (f"{spec.name}: {spec.n_prompts} prompts x {spec.group_size} responses, lengths U[{spec.len_lo},"
             f"{spec.len_hi}], V={spec.V}, bf16 logits {spec.dist}(scale {spec.scale}), mu = FP8-E4M3 "
@@ -147,57 +157,83 @@ def _workload_desc(spec):
 # CPU oracle leg
 # --------------------------------------------------------------------------
 
-def oracle_tokens_per_s(batch, params, rows_budget_s=10.0, max_rows=4096, rng_seed=0):
-    """Time the float64 oracle on a bounded sample: the O(T) stages over the
-    whole batch once, the vocabulary-wide stages (log-softmax statistics and the
-    gradient) on sampled rows until `rows_budget_s` has passed.  Returns
-    (tokens/s extrapolated to the whole batch, description)."""
-    import torch
-
+def _oracle_params(params):
     import oracle as O
+    return O.Params(gamma=params.gamma, C=params.C, clip_eps=params.clip_eps, adv_eps=params.adv_eps)
 
-    T, V = batch.T, batch.V
+
+def _oracle_rows(O, z, ids, mask, op):
+    """The oracle's vocabulary-wide stages on a block of rows: statistics, then
+    the gradient with a representative weight and advantage."""
+    lse, logp, H, _ = O.token_stats(z, ids, mask)
+    r = len(ids)
+    O.loss_grad_logits(z, ids, mask, lse, None, np.ones(r), np.ones(r), np.arange(r + 1),
+                       {"n": np.ones(r, dtype=np.int64), "group": np.zeros(r, dtype=np.int64)},
+                       {"n_valid_seqs": np.array([r])}, {"n_groups_valid": 1, "n_tokens": r}, op)
+
+
+def _oracle_ot_seconds(O, batch, op):
+    """The oracle's O(T) stages over the whole batch; the rollout log-probs stand
+    in for pi's (same cost)."""
     mask = batch.mask.cpu().numpy()
-    ids = batch.ids.cpu().numpy()
     mu = batch.logp_mu.cpu().numpy().astype(np.float64)
     R = batch.rewards.cpu().numpy().astype(np.float64)
     so = batch.seq_offsets.cpu().numpy()
     go = batch.group_offsets.cpu().numpy()
-    op = O.Params(gamma=params.gamma, C=params.C, clip_eps=params.clip_eps, adv_eps=params.adv_eps)
-    rng = np.random.default_rng(rng_seed)
-    rows = rng.permutation(np.flatnonzero(mask))[:max_rows]
-    # vocabulary-wide part on sampled rows (time-boxed)
-    t0 = time.perf_counter()
-    done = 0
-    lse_s = {}
-    block = 16
-    while done < len(rows) and time.perf_counter() - t0 < rows_budget_s:
-        rr = rows[done:done + block]
-        idx = torch.as_tensor(rr, device=batch.logits.device)
-        bits = batch.logits.index_select(0, idx)[:, :V].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
-        tc = time.perf_counter()
-        z = O.bf16_bits_to_f64(bits)
-        lse, logp, H, _ = O.token_stats(z, ids[rr], mask[rr])
-        # gradient of the same rows with a representative weight/advantage
-        O.loss_grad_logits(z, ids[rr], mask[rr], lse, None, np.ones(len(rr)), np.ones(len(rr)),
-                           np.arange(len(rr) + 1), {"n": np.ones(len(rr), dtype=np.int64),
-                                                    "group": np.zeros(len(rr), dtype=np.int64)},
-                           {"n_valid_seqs": np.array([len(rr)])}, {"n_groups_valid": 1, "n_tokens": len(rr)}, op)
-        lse_s[done] = time.perf_counter() - tc
-        done += len(rr)
-    t_rows = sum(lse_s.values())
-    # O(T) part on the whole batch, from the batch's own GPU-independent inputs
     tc = time.perf_counter()
-    # the O(T) stages need pi's log-probs for every token; the rollout log-probs stand in (same cost)
     lr, d, seq, grp, bst, _ = O.seq_discrepancy(mu, mu, mask, so, go)
     adv = O.grpo_advantage(R, go, op)
     w, alpha, st, info, _ = O.controller_step(O.controller_init(op), op, lr, mask, so, go, seq, grp, bst, adv)
     O.loss_coefficients(w, adv, mask, so, seq, grp, bst, op)
-    t_ot = time.perf_counter() - tc
+    return time.perf_counter() - tc
+
+
+def _bf16_rows_f64(O, t, rows, cols):
+    import torch
+    idx = torch.as_tensor(rows, device=t.device)
+    bits = t.index_select(0, idx)[:, :cols].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    return O.bf16_bits_to_f64(bits)
+
+
+def oracle_tokens_per_s(batch, params, rows_budget_s=10.0, max_rows=4096, rng_seed=0, lmhead=False):
+    """Time the float64 oracle on a bounded sample: the O(T) stages over the
+    whole batch once, the vocabulary-wide stages (for the LM-head workload the
+    projection first, then log-softmax statistics and the gradient) on sampled
+    rows until `rows_budget_s` has passed.  Returns (tokens/s extrapolated to
+    the whole batch, description, rows done)."""
+    import oracle as O
+
+    op = _oracle_params(params)
+    mask = batch.mask.cpu().numpy()
+    ids = batch.ids.cpu().numpy()
+    rng = np.random.default_rng(rng_seed)
+    rows = rng.permutation(np.flatnonzero(mask))[:max_rows]
+    if lmhead:
+        # the weight's float64 copy is set-up (a model load), not timed
+        W64 = _bf16_rows_f64(O, batch.weight, np.arange(batch.N), batch.K)
+    t0 = time.perf_counter()
+    done = 0
+    t_rows = 0.0
+    block = 4 if lmhead else 16
+    while done < len(rows) and time.perf_counter() - t0 < rows_budget_s:
+        rr = rows[done:done + block]
+        if lmhead:
+            h = _bf16_rows_f64(O, batch.hidden, rr, batch.K)
+            tc = time.perf_counter()
+            z = O.lmhead_logits(h, W64)
+        else:
+            z = _bf16_rows_f64(O, batch.logits, rr, batch.V)
+            tc = time.perf_counter()
+        _oracle_rows(O, z, ids[rr], mask[rr], op)
+        t_rows += time.perf_counter() - tc
+        done += len(rr)
+    t_ot = _oracle_ot_seconds(O, batch, op)
     n_valid = int(mask.sum())
     per_token = t_rows / max(1, done) + t_ot / max(1, n_valid)
-    desc = (f"float64 numpy oracle, 1 thread: log-softmax statistics + gradient on {done} sampled rows "
-            f"({t_rows:.1f} s) and the O(T) stages on all {n_valid} tokens ({t_ot:.1f} s), extrapolated per token")
+    what = "LM-head projection + log-softmax statistics + gradient" if lmhead else \
+        "log-softmax statistics + gradient"
+    desc = (f"float64 numpy oracle, 1 thread: {what} on {done} sampled rows ({t_rows:.1f} s) and the O(T) stages "
+            f"on all {n_valid} tokens ({t_ot:.1f} s), extrapolated per token")
     return 1.0 / per_token, desc, done
 
 
@@ -209,11 +245,18 @@ def run_reference(args):
 
     import paper_2607_24062_gb300 as acrl
     import workloads as W
-    spec = W.QWEN
+    lmhead = args.workload in ("lmhead", "lmhead_profile")
     dev = torch.device(f"cuda:{local}" if torch.cuda.is_available() else "cpu")
     if dev.type == "cuda":
         torch.cuda.set_device(dev)
-    batch = W.generate(spec, seed=W.seed_for(spec.name), device=dev)
+    if lmhead:
+        spec = _lmhead_spec(W, args.workload)
+        batch = W.generate_lmhead(spec, device=dev)
+        config = {"workload": _lmhead_desc(batch), "M": batch.T, "N": batch.N, "K": batch.K}
+    else:
+        spec = W.SPECS[args.workload]
+        batch = W.generate(spec, seed=W.seed_for(spec.name), device=dev)
+        config = {"workload": _workload_desc(spec), "T": batch.T, "V": batch.V}
     params = acrl.Params()
     vals = []
     t_all = []
@@ -221,15 +264,17 @@ def run_reference(args):
     budget = min(args.ref_seconds, max(1.0, 150.0 / max(1, args.warmup + args.steps)))
     for k in range(args.warmup + args.steps):
         t0 = time.perf_counter()
-        v, desc, n = oracle_tokens_per_s(batch, params, rows_budget_s=budget, max_rows=4096, rng_seed=k)
+        v, desc, n = oracle_tokens_per_s(batch, params, rows_budget_s=budget, max_rows=4096, rng_seed=k,
+                                         lmhead=lmhead)
         t_all.append(time.perf_counter() - t0)
         if k >= args.warmup:
             vals.append(v)
     value = float(np.median(vals))
-    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
-           "steps": args.steps, "warmup": args.warmup, "ms_per_step": float(np.median(t_all[args.warmup:])) * 1e3,
+    out = {"impl": "reference", "metric": LMHEAD_METRIC if lmhead else METRIC, "value": value, "unit": UNIT,
+           "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": float(np.median(t_all[args.warmup:])) * 1e3,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": {"workload": _workload_desc(spec), "T": batch.T, "V": batch.V},
+           "config": config,
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
@@ -425,8 +470,7 @@ def run_lmhead(args):
     build.build()
     dev = torch.device(f"cuda:{local}")
     torch.cuda.set_device(dev)
-    spec = W.LMHEAD if args.workload == "lmhead" else W.small_variant(W.LMHEAD, name="lmhead_profile", n_prompts=2)
-    b = W.generate_lmhead(spec, device=dev)
+    b = W.generate_lmhead(_lmhead_spec(W, args.workload), device=dev)
     p = acrl.Params()
     M, N, K = b.T, b.N, b.K
     stream = torch.cuda.current_stream(dev)
@@ -476,12 +520,11 @@ def run_lmhead(args):
     tf = flop / (gemm_ms / 1e3) / 1e12
     peak, kind = _peak_tflops()
     n_valid = int(b.mask.sum())
-    out = {"metric": "tokens/s fused LM-head projection + logprob + discrepancy + grad at V=151936",
+    out = {"metric": LMHEAD_METRIC,
            "value": n_valid * args.steps / (total_ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "bf16 (tensor cores, fp32 accumulate)", "data": "synthetic",
-           "config": {"workload": f"lmhead: hidden bf16 [{M}, {K}] ~N(0,1), weight bf16 [{N}, {K}] ~N(0, 0.02^2), "
-                                  "mu from E4M3 per-token/per-channel copies", "flags": fl},
+           "config": {"workload": _lmhead_desc(b), "flags": fl},
            "roofline": {"bound": "tensor", "kernel": "acrl_lmhead_logits_stats", "achieved": tf, "peak": peak,
                         "unit": "TFLOP/s", "frac": tf / peak, "traffic": None, "peak_kind": kind,
                         "flop_per_launch": flop, "ms_per_launch": gemm_ms},
@@ -489,6 +532,9 @@ def run_lmhead(args):
                        "acrl_loss_grad_logits": {"ms": grad_ms,
                                                  "GB/s": 4.0 * M * N / (grad_ms / 1e3) / 1e9}},
            "clocks": clocks.summary(), "gpu_launches": 11 * args.steps}
+    if not args.no_cpu:
+        v, desc, _ = oracle_tokens_per_s(b, p, rows_budget_s=args.ref_seconds, lmhead=True)
+        out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
     print(json.dumps(out))
     return 0
 

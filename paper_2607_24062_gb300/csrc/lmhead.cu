@@ -29,10 +29,7 @@
 namespace acrl {
 namespace {
 
-constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
-constexpr int kABytes = kBM * kBK * 2;
-constexpr int kBBytes = kBN * kBK * 2;
-constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kBM = 128, kBN = 256;
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
 constexpr int kBandM = 16;
@@ -41,17 +38,43 @@ constexpr int kBandM = 16;
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kBN >> 3) << 17) |
                             (uint32_t(kBM >> 4) << 24);
 
-struct Barriers {
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
-    uint64_t tfull[2];
-    uint64_t tempty[2];
-    uint64_t mma_done;
-    uint32_t tmem_base;
-    int32_t abort;
+// Shape of the shared-memory ring: K-slab width BK (64 columns = 128-byte
+// rows under the 128-byte swizzle, 32 columns = 64-byte rows under the 64-byte
+// swizzle) and the number of stages.  The loads in flight cover (STAGES - 1)
+// stages of MMA time.  Measured on 32768 x 4096 x 151936: 64 x 4 stages 1574
+// TFLOP/s, 64 x 3 1439; 32 x 6, 8 or 9 stages 1056-1171 whatever the depth (the
+// operand reads of 64-byte-swizzled tiles are the limit there).  A fifth
+// 64-column stage does not fit in shared memory.
+template <int BK, int STAGES>
+struct Ring {
+    static_assert(BK == 32 || BK == 64, "K slab of 32 or 64 bf16 columns");
+    static constexpr int kBK = BK, kStages = STAGES;
+    static constexpr int kRowBytes = BK * 2;
+    static constexpr int kABytes = kBM * kRowBytes;
+    static constexpr int kBBytes = kBN * kRowBytes;
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    // tcgen05 shared-memory descriptor: swizzle code (2 = 128-byte, 4 = 64-byte)
+    // and the stride between 8-row groups
+    static constexpr uint64_t kSwizzleCode = BK == 64 ? 2 : 4;
+    static constexpr uint32_t kGroupStride = 8 * kRowBytes;
+    static constexpr CUtensorMapSwizzle kTmaSwizzle = BK == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    struct Barriers {
+        uint64_t full[STAGES];
+        uint64_t empty[STAGES];
+        uint64_t tfull[2];
+        uint64_t tempty[2];
+        uint64_t mma_done;
+        uint32_t tmem_base;
+        int32_t abort;
+    };
+    // The B stages come first, then the A stages, then the barriers, with a
+    // margin behind them (every descriptor read stays inside the allocation).
+    static constexpr int kMargin = 8192;
+    static constexpr int kSmemBytes = 1024 + STAGES * kStageBytes + int(sizeof(Barriers)) + kMargin;
+    static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
 };
 
-constexpr int kSmemBytes = 1024 + kStages * kStageBytes + int(sizeof(Barriers));
+using LmRing = Ring<64, 4>;
 
 // ---------------------------------------------------------------------------
 // PTX wrappers
@@ -69,12 +92,13 @@ __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence:
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
 // Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with
-// 128-byte swizzling: rows of 128 bytes, 8-row groups 1024 bytes apart.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
-    uint64_t d = uint64_t((addr & 0x3FFFFu) >> 4);  // start address
-    d |= uint64_t(1024 >> 4) << 32;                  // stride between 8-row groups
-    d |= uint64_t(1) << 46;                          // descriptor version of tcgen05
-    d |= uint64_t(2) << 61;                          // 128-byte swizzle
+// the ring's swizzle: rows of BK*2 bytes, 8-row groups 8*BK*2 bytes apart.
+template <class R>
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
+    uint64_t d = uint64_t((addr & 0x3FFFFu) >> 4);            // start address
+    d |= uint64_t(R::kGroupStride >> 4) << 32;                 // stride between 8-row groups
+    d |= uint64_t(1) << 46;                                    // descriptor version of tcgen05
+    d |= R::kSwizzleCode << 61;                                // swizzle mode
     return d;
 }
 
@@ -124,8 +148,10 @@ __device__ __forceinline__ void give_up(volatile int32_t* abort, int32_t* flags)
 // roles
 // ---------------------------------------------------------------------------
 
-__device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t* sA, uint8_t* sB, Barriers* bars,
-                         int m_tiles, int n_tiles, int total, int k_iters, int32_t* flags) {
+template <class R>
+__device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t* sA, uint8_t* sB,
+                         typename R::Barriers* bars, int m_tiles, int n_tiles, int total, int k_iters, int32_t* flags) {
+    constexpr int kStages = R::kStages;
     volatile int32_t* abort = &bars->abort;
     int stage = 0;
     uint32_t phase = 0;
@@ -140,9 +166,9 @@ __device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t
                 ok = false;
                 break;
             }
-            mbar_expect_tx(&bars->full[stage], kStageBytes);
-            tma_load_2d(sA + stage * kABytes, tmA, &bars->full[stage], kk * kBK, m * kBM);
-            tma_load_2d(sB + stage * kBBytes, tmB, &bars->full[stage], kk * kBK, n * kBN);
+            mbar_expect_tx(&bars->full[stage], R::kStageBytes);
+            tma_load_2d(sA + stage * R::kABytes, tmA, &bars->full[stage], kk * R::kBK, m * kBM);
+            tma_load_2d(sB + stage * R::kBBytes, tmB, &bars->full[stage], kk * R::kBK, n * kBN);
             ++issued;
             if (++stage == kStages) {
                 stage = 0;
@@ -157,8 +183,10 @@ __device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t
     }
 }
 
-__device__ void mma_issuer(uint8_t* sA, uint8_t* sB, Barriers* bars, uint32_t tmem, int total, int k_iters,
-                           int32_t* flags) {
+template <class R>
+__device__ void mma_issuer(uint8_t* sA, uint8_t* sB, typename R::Barriers* bars, uint32_t tmem, int total,
+                           int k_iters, int32_t* flags) {
+    constexpr int kStages = R::kStages;
     volatile int32_t* abort = &bars->abort;
     int stage = 0;
     uint32_t phase = 0;
@@ -179,11 +207,11 @@ __device__ void mma_issuer(uint8_t* sA, uint8_t* sB, Barriers* bars, uint32_t tm
                 break;
             }
             tc_fence_after();
-            const uint32_t a0 = smem_u32(sA + stage * kABytes);
-            const uint32_t b0 = smem_u32(sB + stage * kBBytes);
+            const uint32_t a0 = smem_u32(sA + stage * R::kABytes);
+            const uint32_t b0 = smem_u32(sB + stage * R::kBBytes);
 #pragma unroll
-            for (int k16 = 0; k16 < kBK / 16; ++k16)
-                mma_bf16(d, sw128_desc(a0 + k16 * 32), sw128_desc(b0 + k16 * 32), (kk | k16) != 0);
+            for (int k16 = 0; k16 < R::kBK / 16; ++k16)  // 16 columns = 32 bytes along the swizzled row
+                mma_bf16(d, smem_desc<R>(a0 + k16 * 32), smem_desc<R>(b0 + k16 * 32), (kk | k16) != 0);
             mma_commit(&bars->empty[stage]);
             if (++stage == kStages) {
                 stage = 0;
@@ -200,7 +228,8 @@ __device__ void mma_issuer(uint8_t* sA, uint8_t* sB, Barriers* bars, uint32_t tm
     wait_phase(&bars->mma_done, 0, nullptr);
 }
 
-__device__ void epilogue(Barriers* bars, uint32_t tmem, int M, int N, int m_tiles, int n_tiles, int total,
+template <class Bars>
+__device__ void epilogue(Bars* bars, uint32_t tmem, int M, int N, int m_tiles, int n_tiles, int total,
                          acrl_bf16* __restrict__ logits, int64_t ldl, float4* __restrict__ partials, int32_t* flags) {
     volatile int32_t* abort = &bars->abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -257,18 +286,21 @@ __device__ void epilogue(Barriers* bars, uint32_t tmem, int M, int N, int m_tile
     }
 }
 
+template <class R>
 __global__ void __launch_bounds__(kThreads, 1)
     lmhead_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N, int K,
                   acrl_bf16* __restrict__ logits, int64_t ldl, float4* __restrict__ partials, int32_t* flags) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* sA = base;
-    uint8_t* sB = base + kStages * kABytes;
-    Barriers* bars = reinterpret_cast<Barriers*>(base + kStages * kStageBytes);
+    using Barriers = typename R::Barriers;
+    constexpr int kStages = R::kStages;
+    uint8_t* sB = base;
+    uint8_t* sA = base + kStages * R::kBBytes;
+    Barriers* bars = reinterpret_cast<Barriers*>(base + kStages * R::kStageBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m_tiles = (M + kBM - 1) / kBM, n_tiles = (N + kBN - 1) / kBN;
     const int total = m_tiles * n_tiles;
-    const int k_iters = (K + kBK - 1) / kBK;
+    const int k_iters = (K + R::kBK - 1) / R::kBK;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -297,9 +329,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = bars->tmem_base;
 
     if (warp == 0) {
-        if (lane == 0) producer(&tmA, &tmB, sA, sB, bars, m_tiles, n_tiles, total, k_iters, flags);
+        if (lane == 0) producer<R>(&tmA, &tmB, sA, sB, bars, m_tiles, n_tiles, total, k_iters, flags);
     } else if (warp == 1) {
-        if (lane == 0) mma_issuer(sA, sB, bars, tmem, total, k_iters, flags);
+        if (lane == 0) mma_issuer<R>(sA, sB, bars, tmem, total, k_iters, flags);
     } else {
         epilogue(bars, tmem, M, N, m_tiles, n_tiles, total, logits, ldl, partials, flags);
     }
@@ -333,7 +365,8 @@ __global__ void lmhead_merge_kernel(const float4* __restrict__ partials, const a
     row_outputs(acc, mx, logits + int64_t(row) * ldl, N, ids[row], lse, logp, ent, row, flags);
 }
 
-bool encode_map(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows) {
+bool encode_map(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows,
+                uint32_t box_cols, CUtensorMapSwizzle swizzle) {
     void* fn = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
@@ -342,11 +375,36 @@ bool encode_map(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols,
     auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {ld * 2};
-    const cuuint32_t box[2] = {uint32_t(kBK), box_rows};
+    const cuuint32_t box[2] = {box_cols, box_rows};
     const cuuint32_t estr[2] = {1, 1};
     return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Tensor maps, shared-memory opt-in and the persistent launch (one CTA per SM,
+// fewer if there are fewer tiles).  Arguments are checked by the callers.
+template <class R>
+acrl_status launch_lmhead(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t ldh, const acrl_bf16* weight,
+                          int64_t N, int64_t ldw, acrl_bf16* logits, int64_t ldl, float4* partials, int32_t* flags,
+                          cudaStream_t s) {
+    CUtensorMap tmA, tmB;
+    if (!encode_map(&tmA, hidden, uint64_t(M), uint64_t(K), uint64_t(ldh), kBM, R::kBK, R::kTmaSwizzle) ||
+        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN, R::kBK, R::kTmaSwizzle))
+        return ACRL_ERR_CUDA;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return ACRL_ERR_CUDA;
+    if (cudaFuncSetAttribute(lmhead_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, R::kSmemBytes) !=
+        cudaSuccess)
+        return ACRL_ERR_CUDA;
+    const int64_t total = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
+    if (total > kMaxGrid) return ACRL_ERR_INVALID_ARG;
+    const int grid = int(total < sms ? total : sms);
+    lmhead_kernel<R><<<grid, kThreads, R::kSmemBytes, s>>>(tmA, tmB, int(M), int(N), int(K), logits, ldl, partials,
+                                                          flags);
+    return launch_status();
 }
 
 }  // namespace
@@ -370,22 +428,8 @@ extern "C" acrl_status acrl_lmhead_logits_stats(const acrl_bf16* hidden, int64_t
     if (!hidden || !weight || !logits || !partials) return ACRL_ERR_INVALID_ARG;
     if (!aligned16(hidden) || !aligned16(weight) || !aligned16(logits) || !aligned16(partials))
         return ACRL_ERR_INVALID_ARG;
-    CUtensorMap tmA, tmB;
-    if (!encode_map(&tmA, hidden, uint64_t(M), uint64_t(K), uint64_t(ldh), kBM) ||
-        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN))
-        return ACRL_ERR_CUDA;
-    int dev = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-        return ACRL_ERR_CUDA;
-    if (cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess)
-        return ACRL_ERR_CUDA;
-    const int64_t total = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
-    if (total > kMaxGrid) return ACRL_ERR_INVALID_ARG;
-    const int grid = int(total < sms ? total : sms);
-    lmhead_kernel<<<grid, kThreads, kSmemBytes, reinterpret_cast<cudaStream_t>(stream)>>>(
-        tmA, tmB, int(M), int(N), int(K), logits, ldl, reinterpret_cast<float4*>(partials), dev_flags);
-    return launch_status();
+    return launch_lmhead<LmRing>(hidden, M, K, ldh, weight, N, ldw, logits, ldl, reinterpret_cast<float4*>(partials),
+                                 dev_flags, reinterpret_cast<cudaStream_t>(stream));
 }
 
 extern "C" acrl_status acrl_lmhead_merge(const float* partials, const acrl_bf16* logits, int64_t M, int64_t N,
@@ -453,23 +497,13 @@ extern "C" acrl_status acrl_lmhead_stats_noalloc(const acrl_bf16* hidden, int64_
     if (M == 0) return ACRL_OK;
     if (!hidden || !weight || !logits || !ids || !lse || !logp || !entropy) return ACRL_ERR_INVALID_ARG;
     if (!aligned16(hidden) || !aligned16(weight) || !aligned16(logits)) return ACRL_ERR_INVALID_ARG;
-    int dev = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-        return ACRL_ERR_CUDA;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return ACRL_ERR_CUDA;
     float4* partials = noalloc_scratch(dev);
     if (partials == nullptr) return ACRL_ERR_CUDA;
-    CUtensorMap tmA, tmB;
-    if (!encode_map(&tmA, hidden, uint64_t(M), uint64_t(K), uint64_t(ldh), kBM) ||
-        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN))
-        return ACRL_ERR_CUDA;
-    if (cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess)
-        return ACRL_ERR_CUDA;
-    const int64_t total = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
-    const int grid = int(total < sms ? total : sms);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    lmhead_kernel<<<grid, kThreads, kSmemBytes, s>>>(tmA, tmB, int(M), int(N), int(K), logits, ldl, partials,
-                                                      dev_flags);
+    const acrl_status st = launch_lmhead<LmRing>(hidden, M, K, ldh, weight, N, ldw, logits, ldl, partials, dev_flags, s);
+    if (st != ACRL_OK) return st;
     const int threads = 128;
     lmhead_merge_kernel<<<unsigned((M + threads - 1) / threads), threads, 0, s>>>(
         partials, logits, int(M), int(N), ldl, int((N + kBN - 1) / kBN), ids, mask, lse, logp, entropy, dev_flags);
