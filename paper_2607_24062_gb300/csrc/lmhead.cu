@@ -12,7 +12,9 @@
 //              into a TMEM accumulator and commits each stage back to the
 //              producer; two 256-column accumulators alternate between tiles;
 //   warps 2-5  the epilogue: tcgen05.ld of the accumulator (each thread one
-//              row), round to bf16, store the logits, fold the statistics.
+//              row), round to bf16, fold the statistics, and write the logits
+//              through shared memory with TMA bulk tensor stores (32 x 32
+//              blocks, two staging buffers per warp).
 // Tiles are visited in bands of 16 row tiles so that the weight tiles in
 // flight are shared through L2 by the CTAs working on the same band.
 // Every wait on an mbarrier is bounded in time; on expiry the kernel raises
@@ -33,6 +35,10 @@ constexpr int kBM = 128, kBN = 256;
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
 constexpr int kBandM = 16;
+// Output staging: each epilogue warp owns two 32 x 32 bf16 blocks (its 32
+// rows x one 32-column chunk of the accumulator), stored 64-byte-swizzled.
+constexpr int kOutBlockBytes = 32 * 32 * 2;
+constexpr int kOutBytes = 4 * 2 * kOutBlockBytes;
 // Instruction descriptor of tcgen05.mma kind::f16: D f32 (bits 4-5 = 1),
 // A and B bf16 (bits 7-9, 10-12 = 1), both K-major, N/8 at bit 17, M/16 at bit 24.
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kBN >> 3) << 17) |
@@ -67,10 +73,11 @@ struct Ring {
         uint32_t tmem_base;
         int32_t abort;
     };
-    // The B stages come first, then the A stages, then the barriers, with a
-    // margin behind them (every descriptor read stays inside the allocation).
+    // The B stages come first, then the A stages, the output staging blocks
+    // and the barriers, with a margin behind them (every descriptor read stays
+    // inside the allocation).
     static constexpr int kMargin = 8192;
-    static constexpr int kSmemBytes = 1024 + STAGES * kStageBytes + int(sizeof(Barriers)) + kMargin;
+    static constexpr int kSmemBytes = 1024 + STAGES * kStageBytes + kOutBytes + int(sizeof(Barriers)) + kMargin;
     static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
 };
 
@@ -125,6 +132,30 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
         : "r"(taddr));
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+
+__device__ __forceinline__ void st_shared16(uint32_t addr, const uint4& v) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+// Make this thread's shared-memory writes visible to the TMA (async proxy).
+__device__ __forceinline__ void fence_async_shared() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y), "r"(smem_u32(src))
+                 : "memory");
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+
+// Wait until at most N of this thread's bulk stores still read shared memory.
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // ---------------------------------------------------------------------------
 // tile schedule: bands of kBandM row tiles, all column tiles of a band in turn
@@ -229,12 +260,17 @@ __device__ void mma_issuer(uint8_t* sA, uint8_t* sB, typename R::Barriers* bars,
 }
 
 template <class Bars>
-__device__ void epilogue(Bars* bars, uint32_t tmem, int M, int N, int m_tiles, int n_tiles, int total,
-                         acrl_bf16* __restrict__ logits, int64_t ldl, float4* __restrict__ partials, int32_t* flags) {
+__device__ void epilogue(Bars* bars, uint32_t tmem, const CUtensorMap* tmC, uint8_t* sOut, int M, int N, int m_tiles,
+                         int n_tiles, int total, float4* __restrict__ partials, int32_t* flags) {
     volatile int32_t* abort = &bars->abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quarter = warp & 3;  // the TMEM lanes (rows) this warp may read
     const uint32_t lane_off = uint32_t(quarter * 32) << 16;
+    // this warp's two staging blocks; row `lane` at 64 bytes, its 16-byte
+    // pieces permuted by the 64-byte swizzle the output tensor map applies
+    const uint32_t out0 = smem_u32(sOut + (warp - 2) * 2 * kOutBlockBytes) + uint32_t(lane * 64);
+    const uint32_t swz = uint32_t((lane >> 1) & 3);
+    int buf = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
@@ -246,8 +282,8 @@ __device__ void epilogue(Bars* bars, uint32_t tmem, int M, int N, int m_tiles, i
             break;
         }
         tc_fence_after();
-        const int row = m * kBM + quarter * 32 + lane;
-        acrl_bf16* out = logits + int64_t(row) * ldl;
+        const int row0 = m * kBM + quarter * 32;
+        const int row = row0 + lane;
         LseAcc st = lse_empty();
         float mx = -INFINITY;
 #pragma unroll 1
@@ -261,42 +297,54 @@ __device__ void epilogue(Bars* bars, uint32_t tmem, int M, int N, int m_tiles, i
                 if (lane == 0) mbar_arrive(&bars->tempty[acc]);
             }
             const int col0 = n * kBN + c * 32;
-            if (row >= M || col0 >= N) continue;
+            if (col0 >= N) continue;  // the same for the whole warp
             uint4 v[4];
             uint32_t* w = reinterpret_cast<uint32_t*>(v);
 #pragma unroll
             for (int j = 0; j < 16; ++j) w[j] = pack_bf16x2(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
-            if (col0 + 32 <= N) {
-                fold_vectors<4>(st, mx, v);
-                uint4* dst = reinterpret_cast<uint4*>(out + col0);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) st_stream(dst + q, v[q]);
-            } else {
-                const acrl_bf16* h = reinterpret_cast<const acrl_bf16*>(v);
-                for (int j = 0; j < N - col0; ++j) {
-                    fold_scalar(st, mx, bf16_to_float(h[j]));
-                    out[col0 + j] = h[j];
+            if (row < M) {
+                if (col0 + 32 <= N) {
+                    fold_vectors<4>(st, mx, v);
+                } else {
+                    const acrl_bf16* h = reinterpret_cast<const acrl_bf16*>(v);
+                    for (int j = 0; j < N - col0; ++j) fold_scalar(st, mx, bf16_to_float(h[j]));
                 }
             }
+            // stage the block and store it with one TMA copy, which leaves out
+            // the rows at or beyond M and the columns at or beyond N
+            if (lane == 0) bulk_wait_read<1>();  // the store that last read this buffer is done
+            __syncwarp();
+            const uint32_t dst = out0 + uint32_t(buf * kOutBlockBytes);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) st_shared16(dst + ((uint32_t(q) ^ swz) << 4), v[q]);
+            fence_async_shared();
+            __syncwarp();
+            if (lane == 0 && row0 < M)
+                tma_store_2d(tmC, sOut + (warp - 2) * 2 * kOutBlockBytes + buf * kOutBlockBytes, col0, row0);
+            buf ^= 1;
         }
         if (row < M) partials[int64_t(n) * M + row] = make_float4(mx, st.U, st.s0, st.s1);
         __syncwarp();
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1u;
     }
+    if (lane == 0) bulk_wait_all();  // the staging blocks stay valid until every store has completed
+    __syncwarp();
 }
 
 template <class R>
 __global__ void __launch_bounds__(kThreads, 1)
-    lmhead_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N, int K,
-                  acrl_bf16* __restrict__ logits, int64_t ldl, float4* __restrict__ partials, int32_t* flags) {
+    lmhead_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                  const __grid_constant__ CUtensorMap tmC, int M, int N, int K, float4* __restrict__ partials,
+                  int32_t* flags) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     using Barriers = typename R::Barriers;
     constexpr int kStages = R::kStages;
     uint8_t* sB = base;
     uint8_t* sA = base + kStages * R::kBBytes;
-    Barriers* bars = reinterpret_cast<Barriers*>(base + kStages * R::kStageBytes);
+    uint8_t* sOut = base + kStages * R::kStageBytes;
+    Barriers* bars = reinterpret_cast<Barriers*>(sOut + kOutBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m_tiles = (M + kBM - 1) / kBM, n_tiles = (N + kBN - 1) / kBN;
     const int total = m_tiles * n_tiles;
@@ -316,6 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmC)) : "memory");
     }
     if (warp == 2) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&bars->tmem_base)),
@@ -333,7 +382,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         if (lane == 0) mma_issuer<R>(sA, sB, bars, tmem, total, k_iters, flags);
     } else {
-        epilogue(bars, tmem, M, N, m_tiles, n_tiles, total, logits, ldl, partials, flags);
+        epilogue(bars, tmem, &tmC, sOut, M, N, m_tiles, n_tiles, total, partials, flags);
     }
     tc_fence_before();
     __syncthreads();
@@ -388,9 +437,10 @@ template <class R>
 acrl_status launch_lmhead(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t ldh, const acrl_bf16* weight,
                           int64_t N, int64_t ldw, acrl_bf16* logits, int64_t ldl, float4* partials, int32_t* flags,
                           cudaStream_t s) {
-    CUtensorMap tmA, tmB;
+    CUtensorMap tmA, tmB, tmC;
     if (!encode_map(&tmA, hidden, uint64_t(M), uint64_t(K), uint64_t(ldh), kBM, R::kBK, R::kTmaSwizzle) ||
-        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN, R::kBK, R::kTmaSwizzle))
+        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN, R::kBK, R::kTmaSwizzle) ||
+        !encode_map(&tmC, logits, uint64_t(M), uint64_t(N), uint64_t(ldl), 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
         return ACRL_ERR_CUDA;
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -402,8 +452,7 @@ acrl_status launch_lmhead(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t
     const int64_t total = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
     if (total > kMaxGrid) return ACRL_ERR_INVALID_ARG;
     const int grid = int(total < sms ? total : sms);
-    lmhead_kernel<R><<<grid, kThreads, R::kSmemBytes, s>>>(tmA, tmB, int(M), int(N), int(K), logits, ldl, partials,
-                                                          flags);
+    lmhead_kernel<R><<<grid, kThreads, R::kSmemBytes, s>>>(tmA, tmB, tmC, int(M), int(N), int(K), partials, flags);
     return launch_status();
 }
 
