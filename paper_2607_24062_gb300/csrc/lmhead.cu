@@ -192,7 +192,8 @@ __device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t
         int m, n;
         tile_coords(t, m_tiles, n_tiles, m, n);
         for (int kk = 0; kk < k_iters; ++kk) {
-            if (!wait_phase(&bars->empty[stage], phase ^ 1u, abort)) {
+            if (!mbar_try_wait(&bars->empty[stage], phase ^ 1u) &&
+                !wait_phase(&bars->empty[stage], phase ^ 1u, abort)) {
                 give_up(abort, flags);
                 ok = false;
                 break;
@@ -219,6 +220,8 @@ __device__ void mma_issuer(uint8_t* sA, uint8_t* sB, typename R::Barriers* bars,
                            int k_iters, int32_t* flags) {
     constexpr int kStages = R::kStages;
     volatile int32_t* abort = &bars->abort;
+    // descriptors of stage 0; a descriptor advances by (address offset) / 16
+    const uint64_t adesc0 = smem_desc<R>(smem_u32(sA)), bdesc0 = smem_desc<R>(smem_u32(sB));
     int stage = 0;
     uint32_t phase = 0;
     int acc = 0;
@@ -232,17 +235,18 @@ __device__ void mma_issuer(uint8_t* sA, uint8_t* sB, typename R::Barriers* bars,
         tc_fence_after();
         const uint32_t d = tmem + uint32_t(acc * kBN);
         for (int kk = 0; kk < k_iters; ++kk) {
-            if (!wait_phase(&bars->full[stage], phase, abort)) {
+            // the common case (the stage has landed) stays inline; the bounded wait is the slow path
+            if (!mbar_try_wait(&bars->full[stage], phase) && !wait_phase(&bars->full[stage], phase, abort)) {
                 give_up(abort, flags);
                 ok = false;
                 break;
             }
             tc_fence_after();
-            const uint32_t a0 = smem_u32(sA + stage * R::kABytes);
-            const uint32_t b0 = smem_u32(sB + stage * R::kBBytes);
+            const uint64_t ad = adesc0 + uint64_t((stage * R::kABytes) >> 4);
+            const uint64_t bd = bdesc0 + uint64_t((stage * R::kBBytes) >> 4);
 #pragma unroll
-            for (int k16 = 0; k16 < R::kBK / 16; ++k16)  // 16 columns = 32 bytes along the swizzled row
-                mma_bf16(d, smem_desc<R>(a0 + k16 * 32), smem_desc<R>(b0 + k16 * 32), (kk | k16) != 0);
+            for (int k16 = 0; k16 < R::kBK / 16; ++k16)  // 16 columns = 32 bytes = 2 descriptor units
+                mma_bf16(d, ad + uint64_t(2 * k16), bd + uint64_t(2 * k16), (kk | k16) != 0);
             mma_commit(&bars->empty[stage]);
             if (++stage == kStages) {
                 stage = 0;
