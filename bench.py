@@ -535,7 +535,7 @@ def run_lmhead(args):
            "kernels": {"acrl_lmhead_logits_stats": {"ms": gemm_ms, "TFLOP/s": tf},
                        "acrl_loss_grad_logits": {"ms": grad_ms,
                                                  "GB/s": 4.0 * M * N / (grad_ms / 1e3) / 1e9}},
-           "clocks": clocks.summary(), "gpu_launches": 11 * args.steps}
+           "clocks": clocks.summary(), "gpu_launches": 10 * args.steps}
     if not args.no_cpu:
         v, desc, _ = oracle_tokens_per_s(b, p, rows_budget_s=args.ref_seconds, lmhead=True)
         out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
