@@ -39,7 +39,10 @@ def _check_logits(got_bf16, ref, abs_sum, K, what="logits"):
     assert np.mean(got == ref) > 0.99
 
 
-@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (200, 1000, 328), (384, 2304, 4096), (130, 151936, 64)])
+# also: one row and a vocabulary narrower than a 32-column store block; an odd number of row tiles (the second
+# CTA of the last cluster has no rows) with a ragged K; K narrower than one 64-column slab
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (200, 1000, 328), (384, 2304, 4096), (130, 151936, 64),
+                                   (1, 8, 64), (257, 520, 72), (5, 40, 8)])
 def test_lmhead_small_shapes(M, N, K):
     gen = torch.Generator(device=DEV).manual_seed(M * 7 + N + K)
     H = torch.randn((M, K), generator=gen, device=DEV).to(torch.bfloat16)
