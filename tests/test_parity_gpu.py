@@ -473,3 +473,44 @@ def test_fully_masked_batch():
     assert torch.all(step.grad[:, :b.V] == 0) and float(step.loss) == 0.0
     assert int(step.batch_host()["n_tokens"]) == 0
     assert api.read_flags(step.flags) == acrl.FLAG_X_NONPOS
+
+
+def test_exchange_hook_as_two_identical_ranks():
+    """The exchange hook sees the device bytes of the batch statistics between
+    the discrepancy statistics and the controller.  An all-reduce over two
+    ranks that hold the same batch doubles the three exchanged sums; doing
+    that here must give the oracle's result on the batch concatenated with
+    itself (one global X, the loss normalised by the global prompt count),
+    restricted to the first copy."""
+    from paper_2607_24062_gb300 import distributed as D
+    spec = W.small_variant(W.GRPO, name="tworanks", n_prompts=3, group_size=4, len_lo=10, len_hi=120, V=3000,
+                           perturb_frac=0.4, perturb_std=0.3)
+    b = _gen(spec, seed=13)
+
+    def as_two_ranks(buf):
+        for name, dt in (("n_tokens", torch.int64), ("n_groups_valid", torch.int32), ("Y_sum", torch.float64)):
+            D._field(buf, name, dt).mul_(2)
+
+    params = acrl.Params()
+    step = acrl.AcrlStep.for_batch(b, params)
+    step.run_batch(b, exchange=as_two_ranks)
+    torch.cuda.synchronize()
+    h = _host_inputs(b)
+    op = oracle_params(params)
+    z = rows_f64(b.logits, np.arange(b.T), b.V)
+    T, S = b.T, b.S
+    cat = np.concatenate
+    so2, go2 = cat([h["so"], h["so"][1:] + T]), cat([h["go"], h["go"][1:] + S]).astype(np.int32)
+    ids2, mask2 = cat([h["ids"], h["ids"]]), cat([h["mask"], h["mask"]])
+    res = O.step(cat([z, z]), ids2, mask2, cat([h["mu"], h["mu"]]), cat([h["R"], h["R"]]), so2, go2, op)
+    gb = step.batch_host()
+    assert int(gb["n_tokens"]) == res.batch["n_tokens"] and int(gb["n_groups_valid"]) == res.batch["n_groups_valid"]
+    assert_close_rel(step.state_host()["X"], res.state.X, floor=1e-12, what="X")
+    assert_close_rel(host(step.weight), res.weight[:T], floor=1e-7, what="weight")
+    coef2 = O.loss_coefficients(res.weight, res.adv, mask2, so2, res.seq, res.grp, res.batch, op)
+    assert_close_rel(host(step.coef), coef2[:T], floor=1e-12, what="coef")
+    assert_close_rel(host(step.token_loss), res.token_loss[:T], floor=1e-12, what="token_loss")
+    assert_loss(float(step.loss), 0.5 * res.loss, res.token_loss[:T])
+    assert_grad_rows(grad_rows(step.grad, np.arange(T), b.V), res.grad[:T], coef2[:T], h["ids"])
+    # without the exchange every coefficient would be twice as large
+    assert np.any(np.abs(coef2[:T]) > 0)
