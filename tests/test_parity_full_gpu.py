@@ -118,8 +118,8 @@ def test_full_size_workload(name):
     rows, whole = _sample_rows(b, rng)
     _check_rows(step, b, rows, ref, op)
     _oracle_chain_on_whole(step, b, whole, op)
-    # cached-old path (lse recomputed inside the gradient call; at V = 151,936 a cluster of CTAs keeps each row
-    # in shared memory) on the first 4,096 rows: the same gradient as the streaming call
+    # cached-old path (lse recomputed inside the gradient call by a first sweep over each row) on the first
+    # 4,096 rows: the same gradient as the streaming call
     R = min(4096, b.T)
     g2, tl2, _ = api.loss_grad_logits(b.logits[:R], b.ids[:R], b.mask[:R], None, step.logp[:R], step.coef[:R],
                                       p.clip_eps, V=b.V)
@@ -135,6 +135,18 @@ def test_full_size_workload(name):
         mr = masked[:: max(1, len(masked) // 64)]
         assert np.all(grad_rows(step.grad, mr, b.V) == 0)
         assert np.all(host(step.logp)[mr] == 0) and np.all(host(step.entropy)[mr] == 0)
+    # the whole step again from a fresh controller: every output bit for bit the same (fixed reduction orders,
+    # no atomics)
+    del g2, tl2
+    step2 = acrl.AcrlStep.for_batch(b, p)
+    step2.run_batch(b)
+    torch.cuda.synchronize()
+    for name in ("lse", "logp", "entropy", "weight", "coef", "alpha", "adv", "token_loss", "loss", "state"):
+        assert torch.equal(getattr(step, name), getattr(step2, name)), name
+    assert torch.equal(step.disc.batch, step2.disc.batch) and torch.equal(step.disc.seq, step2.disc.seq)
+    for r0 in range(0, b.T, 8192):
+        r1 = min(b.T, r0 + 8192)
+        assert torch.equal(step.grad[r0:r1].view(torch.int16), step2.grad[r0:r1].view(torch.int16)), (r0, r1)
 
 
 def test_long_workload_chunked():
