@@ -12,7 +12,8 @@
  * Conventions shared by every call:
  *   - Pointers documented "device" must be device memory of the current CUDA
  *     device (or managed memory).  The caller owns every buffer; the library
- *     allocates nothing and keeps no global state.
+ *     allocates nothing and keeps no global state, except the fixed scratch
+ *     array of acrl_lmhead_stats_noalloc (documented there).
  *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL is the
  *     legacy default stream) except acrl_read_flags, which synchronises it.
  *   - Problems visible on the host (null required pointers, negative sizes,
