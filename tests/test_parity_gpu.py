@@ -514,3 +514,31 @@ def test_exchange_hook_as_two_identical_ranks():
     assert_grad_rows(grad_rows(step.grad, np.arange(T), b.V), res.grad[:T], coef2[:T], h["ids"])
     # without the exchange every coefficient would be twice as large
     assert np.any(np.abs(coef2[:T]) > 0)
+
+
+def test_autograd_loss_through_an_lm_head():
+    """acrl_loss as a torch.autograd node: loss.backward() delivers the
+    kernel's dL/dlogits (bit for bit, and scaled by the incoming gradient),
+    and it flows on into an upstream bf16 projection like any other grad."""
+    spec = W.small_variant(W.GRPO, name="autograd", n_prompts=2, group_size=4, len_lo=20, len_hi=90, V=2048)
+    b = _gen(spec, seed=21)
+    step = acrl.AcrlStep.for_batch(b, acrl.Params())
+    x = b.logits[:, :b.V].detach().requires_grad_(True)
+    loss = acrl.acrl_loss(step, x, b.ids, b.mask, b.logp_mu, b.rewards, b.seq_offsets, b.group_offsets)
+    loss.backward()
+    torch.cuda.synchronize()
+    assert torch.equal(x.grad.view(torch.int16), step.grad[:, :b.V].view(torch.int16))
+    assert float(loss.detach()) == float(step.loss)
+    x.grad = None
+    (2.0 * acrl.acrl_loss(step, x, b.ids, b.mask, b.logp_mu, b.rewards, b.seq_offsets, b.group_offsets)).backward()
+    assert torch.equal(x.grad.float(), 2.0 * step.grad[:, :b.V].float())
+    # an LM head upstream: logits = h W^T in bf16; W's gradient is g^T h
+    K = 64
+    gen = torch.Generator(device=DEV).manual_seed(5)
+    h = torch.randn((b.T, K), generator=gen, device=DEV).to(torch.bfloat16)
+    Wt = (0.1 * torch.randn((b.V, K), generator=gen, device=DEV)).to(torch.bfloat16).requires_grad_(True)
+    logits = h @ Wt.t()
+    step2 = acrl.AcrlStep(b.T, b.V, b.V, b.S, b.Gn, acrl.Params())
+    acrl.acrl_loss(step2, logits, b.ids, b.mask, b.logp_mu, b.rewards, b.seq_offsets, b.group_offsets).backward()
+    ref = step2.grad.float().t() @ h.float()
+    assert torch.allclose(Wt.grad.float(), ref, rtol=2e-2, atol=1e-6 + 2e-2 * float(ref.abs().max()))
