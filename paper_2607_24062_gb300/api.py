@@ -21,10 +21,39 @@ def _ptr(t: torch.Tensor | None) -> int | None:
     return None if t is None else t.data_ptr()
 
 
-def _stream(stream) -> int | None:
-    if stream is None:
-        stream = torch.cuda.current_stream()
-    return stream.cuda_stream
+def _one_device(tensors) -> torch.device:
+    """The GPU every buffer of one call lives on (they must agree)."""
+    dev = None
+    for t in tensors:
+        if t is None:
+            continue
+        if dev is None:
+            dev = t.device
+        elif t.device != dev:
+            raise AcrlError(f"buffers on {dev} and {t.device}: every buffer of a call must be on one GPU")
+    if dev is None or dev.type != "cuda":
+        raise AcrlError("expected CUDA tensors")
+    return dev
+
+
+def _call(name: str, tensors, stream, *args) -> None:
+    """Call entry point `name` with `args` followed by the stream, on the GPU
+    that holds `tensors` (the stream defaults to that GPU's current stream)."""
+    dev = _one_device(tensors)
+    if stream is not None and stream.device != dev:
+        raise AcrlError(f"{name}: stream on {stream.device}, buffers on {dev}")
+    fn = getattr(lib(), name)
+    if dev.index == torch.cuda.current_device():
+        s = torch.cuda.current_stream(dev) if stream is None else stream
+        check(fn(*args, s.cuda_stream), name)
+        return
+    with torch.cuda.device(dev):
+        s = torch.cuda.current_stream(dev) if stream is None else stream
+        check(fn(*args, s.cuda_stream), name)
+
+
+def _flags(flags, dev):
+    return new_flags(dev) if flags is None else _need(flags, torch.int32, 1, "flags")
 
 
 def _need(t: torch.Tensor, dtype, n: int | None, name: str):
@@ -77,9 +106,9 @@ def token_stats(logits, ids, mask=None, *, V=None, lse=None, logp=None, entropy=
     logp = torch.empty(T, dtype=torch.float32, device=dev) if logp is None else _need(logp, torch.float32, T, "logp")
     entropy = torch.empty(T, dtype=torch.float32, device=dev) if entropy is None else \
         _need(entropy, torch.float32, T, "entropy")
-    flags = new_flags(dev) if flags is None else flags
-    check(lib().acrl_token_stats(_ptr(logits), T, V, ld, _ptr(ids), _ptr(mask), _ptr(lse), _ptr(logp),
-                                 _ptr(entropy), _ptr(flags), _stream(stream)), "acrl_token_stats")
+    flags = _flags(flags, dev)
+    _call("acrl_token_stats", (logits, ids, mask, lse, logp, entropy, flags), stream, _ptr(logits), T, V, ld,
+          _ptr(ids), _ptr(mask), _ptr(lse), _ptr(logp), _ptr(entropy), _ptr(flags))
     return lse, logp, entropy
 
 
@@ -120,11 +149,11 @@ def seq_discrepancy(logp_pi, logp_mu, mask, seq_offsets, group_offsets, entropy=
         out = Discrepancy(torch.empty(T, dtype=torch.float32, device=dev), torch.empty(T, dtype=torch.float32, device=dev),
                           struct_buffer(SEQ_DTYPE, S, dev), struct_buffer(GRP_DTYPE, Gn, dev),
                           struct_buffer(BATCH_DTYPE, 1, dev), S, Gn)
-    flags = new_flags(dev) if flags is None else flags
-    check(lib().acrl_seq_discrepancy(_ptr(logp_pi), _ptr(logp_mu), _ptr(mask), T, _ptr(seq_offsets), S,
-                                     _ptr(group_offsets), Gn, _ptr(entropy), _ptr(out.lr), _ptr(out.d), _ptr(out.seq),
-                                     _ptr(out.grp), _ptr(out.batch), _ptr(flags), _stream(stream)),
-          "acrl_seq_discrepancy")
+    flags = _flags(flags, dev)
+    _call("acrl_seq_discrepancy", (logp_pi, logp_mu, mask, seq_offsets, group_offsets, entropy, out.lr, out.d,
+                                   out.seq, out.grp, out.batch, flags), stream,
+          _ptr(logp_pi), _ptr(logp_mu), _ptr(mask), T, _ptr(seq_offsets), S, _ptr(group_offsets), Gn, _ptr(entropy),
+          _ptr(out.lr), _ptr(out.d), _ptr(out.seq), _ptr(out.grp), _ptr(out.batch), _ptr(flags))
     return out
 
 
@@ -135,16 +164,17 @@ def grpo_advantage(rewards, group_offsets, params: Params, *, adv=None, flags=No
     _need(rewards, torch.float32, S, "rewards")
     _need(group_offsets, torch.int32, Gn + 1, "group_offsets")
     adv = torch.empty(S, dtype=torch.float32, device=rewards.device) if adv is None else _need(adv, torch.float32, S, "adv")
-    flags = new_flags(rewards.device) if flags is None else flags
-    check(lib().acrl_grpo_advantage(_ptr(rewards), _ptr(group_offsets), Gn, S, ctypes.byref(params), _ptr(adv),
-                                    _ptr(flags), _stream(stream)), "acrl_grpo_advantage")
+    flags = _flags(flags, rewards.device)
+    _call("acrl_grpo_advantage", (rewards, group_offsets, adv, flags), stream, _ptr(rewards), _ptr(group_offsets), Gn,
+          S, ctypes.byref(params), _ptr(adv), _ptr(flags))
     return adv
 
 
 def controller_init(params: Params, state=None, device=None, stream=None) -> torch.Tensor:
     """acrl_controller_init; allocates the 48-byte device state if not given."""
     state = struct_buffer(STATE_DTYPE, 1, device) if state is None else state
-    check(lib().acrl_controller_init(_ptr(state), ctypes.byref(params), _stream(stream)), "acrl_controller_init")
+    _need(state, torch.uint8, STATE_DTYPE.itemsize, "state")
+    _call("acrl_controller_init", (state,), stream, _ptr(state), ctypes.byref(params))
     return state
 
 
@@ -181,12 +211,13 @@ def controller_step(state, params: Params, disc: Discrepancy, mask, seq_offsets,
     _need(adv, torch.float32, disc.S, "adv")
     _opt(mask, torch.uint8, T, "mask")
     _opt(ent_coef, torch.float32, T, "ent_coef")
-    flags = new_flags(dev) if flags is None else flags
-    check(lib().acrl_controller_step(_ptr(state), ctypes.byref(params), _ptr(disc.lr), _ptr(mask), T,
-                                     _ptr(seq_offsets), disc.S, _ptr(group_offsets), disc.Gn, _ptr(disc.seq),
-                                     _ptr(disc.grp), _ptr(disc.batch), _ptr(adv), _ptr(weight), _ptr(coef),
-                                     _ptr(alpha), _ptr(ent_coef), _ptr(flags), _stream(stream)),
-          "acrl_controller_step")
+    _need(state, torch.uint8, STATE_DTYPE.itemsize, "state")
+    flags = _flags(flags, dev)
+    _call("acrl_controller_step", (state, disc.lr, mask, seq_offsets, group_offsets, disc.seq, disc.grp, disc.batch,
+                                   adv, weight, coef, alpha, ent_coef, flags), stream,
+          _ptr(state), ctypes.byref(params), _ptr(disc.lr), _ptr(mask), T, _ptr(seq_offsets), disc.S,
+          _ptr(group_offsets), disc.Gn, _ptr(disc.seq), _ptr(disc.grp), _ptr(disc.batch), _ptr(adv), _ptr(weight),
+          _ptr(coef), _ptr(alpha), _ptr(ent_coef), _ptr(flags))
     return weight, coef, alpha
 
 
@@ -212,11 +243,11 @@ def loss_grad_logits(logits, ids, mask, lse, old_logp, coef, clip_eps: float, *,
     token_loss = torch.empty(T, dtype=torch.float32, device=dev) if token_loss is None else \
         _need(token_loss, torch.float32, T, "token_loss")
     loss = torch.empty(1, dtype=torch.float32, device=dev) if loss is None else _need(loss, torch.float32, 1, "loss")
-    flags = new_flags(dev) if flags is None else flags
-    check(lib().acrl_loss_grad_logits(_ptr(logits), T, V, ld, _ptr(ids), _ptr(mask), _ptr(lse), _ptr(old_logp),
-                                      _ptr(coef), _ptr(entropy), _ptr(ent_coef), float(clip_eps), _ptr(grad),
-                                      _ptr(token_loss), _ptr(loss), _ptr(flags), _stream(stream)),
-          "acrl_loss_grad_logits")
+    flags = _flags(flags, dev)
+    _call("acrl_loss_grad_logits", (logits, ids, mask, lse, old_logp, coef, entropy, ent_coef, grad, token_loss, loss,
+                                    flags), stream,
+          _ptr(logits), T, V, ld, _ptr(ids), _ptr(mask), _ptr(lse), _ptr(old_logp), _ptr(coef), _ptr(entropy),
+          _ptr(ent_coef), float(clip_eps), _ptr(grad), _ptr(token_loss), _ptr(loss), _ptr(flags))
     return grad, token_loss, loss
 
 
@@ -224,8 +255,9 @@ def reduce_loss(token_loss, *, loss=None, stream=None):
     """acrl_reduce_loss."""
     T = token_loss.numel()
     _need(token_loss, torch.float32, T, "token_loss")
-    loss = torch.empty(1, dtype=torch.float32, device=token_loss.device) if loss is None else loss
-    check(lib().acrl_reduce_loss(_ptr(token_loss), T, _ptr(loss), _stream(stream)), "acrl_reduce_loss")
+    loss = torch.empty(1, dtype=torch.float32, device=token_loss.device) if loss is None else \
+        _need(loss, torch.float32, 1, "loss")
+    _call("acrl_reduce_loss", (token_loss, loss), stream, _ptr(token_loss), T, _ptr(loss))
     return loss
 
 
@@ -251,11 +283,11 @@ def lmhead_logits_stats(hidden, weight, *, N=None, logits=None, partials=None, f
     nbytes = lmhead_workspace_bytes(M, N)
     if partials is None:
         partials = torch.empty(max(1, nbytes // 4), dtype=torch.float32, device=dev)
-    elif partials.numel() * 4 < nbytes:
-        raise AcrlError("partials: workspace too small")
-    flags = new_flags(dev) if flags is None else flags
-    check(lib().acrl_lmhead_logits_stats(_ptr(hidden), M, K, ldh, _ptr(weight), N, ldw, _ptr(logits), ldl,
-                                         _ptr(partials), _ptr(flags), _stream(stream)), "acrl_lmhead_logits_stats")
+    else:
+        _need(partials, torch.float32, (nbytes + 3) // 4, "partials")
+    flags = _flags(flags, dev)
+    _call("acrl_lmhead_logits_stats", (hidden, weight, logits, partials, flags), stream, _ptr(hidden), M, K, ldh,
+          _ptr(weight), N, ldw, _ptr(logits), ldl, _ptr(partials), _ptr(flags))
     return logits, partials
 
 
@@ -271,16 +303,18 @@ def lmhead_merge(partials, logits, ids, mask=None, *, N=None, lse=None, logp=Non
     logp = torch.empty(M, dtype=torch.float32, device=dev) if logp is None else _need(logp, torch.float32, M, "logp")
     entropy = torch.empty(M, dtype=torch.float32, device=dev) if entropy is None else \
         _need(entropy, torch.float32, M, "entropy")
-    flags = new_flags(dev) if flags is None else flags
-    check(lib().acrl_lmhead_merge(_ptr(partials), _ptr(logits), M, N, ldl, _ptr(ids), _ptr(mask), _ptr(lse),
-                                  _ptr(logp), _ptr(entropy), _ptr(flags), _stream(stream)), "acrl_lmhead_merge")
+    _need(partials, torch.float32, (lmhead_workspace_bytes(M, N) + 3) // 4, "partials")
+    flags = _flags(flags, dev)
+    _call("acrl_lmhead_merge", (partials, logits, ids, mask, lse, logp, entropy, flags), stream, _ptr(partials),
+          _ptr(logits), M, N, ldl, _ptr(ids), _ptr(mask), _ptr(lse), _ptr(logp), _ptr(entropy), _ptr(flags))
     return lse, logp, entropy
 
 
 def read_flags(flags, stream=None) -> int:
     """acrl_read_flags (synchronises the stream)."""
     host = ctypes.c_int32(0)
-    check(lib().acrl_read_flags(_ptr(flags), ctypes.byref(host), _stream(stream)), "acrl_read_flags")
+    _need(flags, torch.int32, 1, "flags")
+    _call("acrl_read_flags", (flags,), stream, _ptr(flags), ctypes.byref(host))
     return int(host.value)
 
 

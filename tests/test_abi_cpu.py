@@ -78,3 +78,18 @@ def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(_abi, "_LIB", None)
     with pytest.raises(_abi.AcrlError):
         _abi.lib()
+
+
+def test_binding_rejects_buffers_on_different_devices():
+    """Every buffer of one call must be on one GPU: the binding refuses a mix
+    before any pointer reaches the library (checked here with host and meta
+    tensors, so no GPU is needed)."""
+    import torch
+    from paper_2607_24062_gb300 import api
+    a, b = torch.empty(4), torch.empty(4, device="meta")
+    with pytest.raises(api.AcrlError, match="one GPU"):
+        api._one_device((a, None, b))
+    with pytest.raises(api.AcrlError, match="CUDA"):
+        api._one_device((a, a))
+    with pytest.raises(api.AcrlError, match="CUDA"):
+        api._one_device((None,))
