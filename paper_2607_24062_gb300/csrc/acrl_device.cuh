@@ -164,4 +164,37 @@ __device__ __forceinline__ T block_max(T v, T* scratch) {
     return r;
 }
 
+// CTA-wide sums of N doubles and the maximum of one more, in the order of
+// block_sum / block_max (a butterfly inside each warp, then the warps in
+// order), with a single shared-memory exchange.  The results are valid in
+// thread 0 only: the cross-warp pass runs there alone (fp64 is a narrow pipe
+// on this part, so the other threads skip it).  `scratch` holds
+// NWARPS * (N + 1) doubles.  Contains __syncthreads(): call from all threads.
+template <int NWARPS, int N>
+__device__ __forceinline__ void block_sums_max0(double (&v)[N], double& mx, double* scratch) {
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) {
+#pragma unroll
+        for (int k = 0; k < N; ++k) v[k] += __shfl_xor_sync(0xffffffffu, v[k], m);
+        mx = fmax(mx, __shfl_xor_sync(0xffffffffu, mx, m));
+    }
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    if (lane == 0) {
+#pragma unroll
+        for (int k = 0; k < N; ++k) scratch[wid * (N + 1) + k] = v[k];
+        scratch[wid * (N + 1) + N] = mx;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+#pragma unroll
+        for (int k = 0; k < N; ++k) v[k] = 0.0;
+        mx = scratch[N];
+        for (int w = 0; w < NWARPS; ++w) {
+#pragma unroll
+            for (int k = 0; k < N; ++k) v[k] += scratch[w * (N + 1) + k];
+            mx = fmax(mx, scratch[w * (N + 1) + N]);
+        }
+    }
+}
+
 }  // namespace acrl

@@ -252,11 +252,11 @@ __global__ void __launch_bounds__(THREADS) loss_grad_warp(
 // Scalar loss: sum of token losses in a fixed order.  Each thread adds float4
 // groups (four values in fp32) into two alternating fp64 accumulators, so the
 // loads pipeline and the fp64 adds are a quarter of the values; then a fixed
-// CTA tree in fp64.
+// CTA tree in fp64 whose cross-warp pass runs in thread 0 alone.
 constexpr int kSumThreads = 1024;
 __global__ void __launch_bounds__(kSumThreads) loss_sum_kernel(const float* __restrict__ tl, int64_t T,
                                                                float* __restrict__ loss) {
-    __shared__ double sh[kSumThreads / 32];
+    __shared__ double sh[kSumThreads / 32 * 2];
     double s0 = 0.0, s1 = 0.0;
     const bool vec = (reinterpret_cast<uintptr_t>(tl) & 15u) == 0;
     const int64_t n4 = vec ? T / 4 : 0;
@@ -273,8 +273,9 @@ __global__ void __launch_bounds__(kSumThreads) loss_sum_kernel(const float* __re
         s0 += double((a.x + a.y) + (a.z + a.w));
     }
     for (int64_t j = 4 * n4 + threadIdx.x; j < T; j += kSumThreads) s1 += tl[j];
-    double s = block_sum<double, kSumThreads / 32>(s0 + s1, sh);
-    if (threadIdx.x == 0) *loss = float(s);
+    double total[1] = {s0 + s1}, unused = 0.0;
+    block_sums_max0<kSumThreads / 32, 1>(total, unused, sh);
+    if (threadIdx.x == 0) *loss = float(total[0]);
 }
 
 template <bool RECOMPUTE, bool ENT>

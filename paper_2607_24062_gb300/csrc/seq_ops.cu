@@ -46,9 +46,7 @@ __global__ void __launch_bounds__(kSeqThreads) seq_stats_kernel(
     const float* __restrict__ entropy, float* __restrict__ lr, float* __restrict__ d, acrl_seq_stats* seq,
     int32_t* flags) {
     constexpr int NW = kSeqThreads / 32;
-    __shared__ double sh_d[NW];
-    __shared__ float sh_f[NW];
-    __shared__ int sh_i[NW];
+    __shared__ double sh[NW * 6];
     const int i = blockIdx.x;
     int64_t lo, hi;
     if (!seq_range(so, i, T, lo, hi)) {
@@ -75,12 +73,14 @@ __global__ void __launch_bounds__(kSeqThreads) seq_stats_kernel(
         lr[t] = l;
         d[t] = dd;
     }
-    n = block_sum<int, NW>(n, sh_i);
-    sd = block_sum<double, NW>(sd, sh_d);
-    sd2 = block_sum<double, NW>(sd2, sh_d);
-    slr = block_sum<double, NW>(slr, sh_d);
-    sH = block_sum<double, NW>(sH, sh_d);
-    mxd = block_max<float, NW>(mxd, sh_f);
+    double v[5] = {double(n), sd, sd2, slr, sH}, mx = mxd;
+    block_sums_max0<NW, 5>(v, mx, sh);
+    n = int(v[0]);
+    sd = v[1];
+    sd2 = v[2];
+    slr = v[3];
+    sH = v[4];
+    mxd = float(mx);
     if (threadIdx.x == 0) {
         acrl_seq_stats s;
         s.n = n;
@@ -103,9 +103,7 @@ __global__ void __launch_bounds__(kFinThreads) seq_finalize_kernel(
     int64_t T, const int64_t* __restrict__ so, int S, const int32_t* __restrict__ goff, int Gn,
     const acrl_seq_stats* __restrict__ seq, acrl_group_stats* grp, acrl_batch_stats* batch, int32_t* flags) {
     constexpr int NW = kFinThreads / 32;
-    __shared__ double sh_d[NW];
-    __shared__ long long sh_l[NW];
-    __shared__ int sh_i[NW];
+    __shared__ double sh[NW * 9];
     bool bad = false;
     for (int i = threadIdx.x; i < S; i += kFinThreads) bad |= so[i] > so[i + 1];
     for (int g = threadIdx.x; g < Gn; g += kFinThreads) bad |= goff[g] > goff[g + 1];
@@ -153,15 +151,17 @@ __global__ void __launch_bounds__(kFinThreads) seq_finalize_kernel(
         slr += s.sum_lr;
         dmax = fmax(dmax, double(s.max_d));
     }
-    qv = block_sum<int, NW>(qv, sh_i);
-    ysum = block_sum<double, NW>(ysum, sh_d);
-    N = block_sum<long long, NW>(N, sh_l);
-    sv = block_sum<int, NW>(sv, sh_i);
-    sd = block_sum<double, NW>(sd, sh_d);
-    sd2 = block_sum<double, NW>(sd2, sh_d);
-    sH = block_sum<double, NW>(sH, sh_d);
-    slr = block_sum<double, NW>(slr, sh_d);
-    dmax = block_max<double, NW>(dmax, sh_d);
+    // counts travel as doubles: exact below 2^53
+    double v[8] = {double(qv), ysum, double(N), double(sv), sd, sd2, sH, slr};
+    block_sums_max0<NW, 8>(v, dmax, sh);
+    qv = int(v[0]);
+    ysum = v[1];
+    N = (long long)v[2];
+    sv = int(v[3]);
+    sd = v[4];
+    sd2 = v[5];
+    sH = v[6];
+    slr = v[7];
     if (threadIdx.x == 0) {
         acrl_batch_stats b = *batch;
         b.n_tokens = N;
@@ -305,8 +305,7 @@ __global__ void __launch_bounds__(kSeqThreads) controller_weights_kernel(
     const acrl_batch_stats* __restrict__ batch, const float* __restrict__ adv, float* __restrict__ weight,
     float* __restrict__ coef, float* __restrict__ ent_coef) {
     constexpr int NW = kSeqThreads / 32;
-    __shared__ double sh_d[NW];
-    __shared__ int sh_i[NW];
+    __shared__ double sh[NW * 3];
     const int i = blockIdx.x;
     int64_t lo, hi;
     if (!seq_range(so, i, T, lo, hi)) lo = hi = 0;
@@ -346,8 +345,10 @@ __global__ void __launch_bounds__(kSeqThreads) controller_weights_kernel(
         coef[t] = w * scale;
         if (ent_coef) ent_coef[t] = m ? escale : 0.f;
     }
-    nt = block_sum<int, NW>(nt, sh_i);
-    sw = block_sum<double, NW>(sw, sh_d);
+    double v[2] = {double(nt), sw}, unused = 0.0;
+    block_sums_max0<NW, 2>(v, unused, sh);
+    nt = int(v[0]);
+    sw = v[1];
     if (threadIdx.x == 0) {
         seq[i].n_trunc = nt;
         seq[i].sum_w = sw;
@@ -358,8 +359,7 @@ __global__ void __launch_bounds__(kSeqThreads) controller_weights_kernel(
 __global__ void __launch_bounds__(kFinThreads) controller_finalize_kernel(int S, const acrl_seq_stats* __restrict__ seq,
                                                                           acrl_batch_stats* batch) {
     constexpr int NW = kFinThreads / 32;
-    __shared__ double sh_d[NW];
-    __shared__ long long sh_l[NW];
+    __shared__ double sh[NW * 4];
     long long nt = 0;
     double sw = 0.0, sa = 0.0;
     for (int i = threadIdx.x; i < S; i += kFinThreads) {
@@ -367,9 +367,11 @@ __global__ void __launch_bounds__(kFinThreads) controller_finalize_kernel(int S,
         sw += seq[i].sum_w;
         if (seq[i].n > 0) sa += seq[i].alpha;
     }
-    nt = block_sum<long long, NW>(nt, sh_l);
-    sw = block_sum<double, NW>(sw, sh_d);
-    sa = block_sum<double, NW>(sa, sh_d);
+    double v[3] = {double(nt), sw, sa}, unused = 0.0;
+    block_sums_max0<NW, 3>(v, unused, sh);
+    nt = (long long)v[0];
+    sw = v[1];
+    sa = v[2];
     if (threadIdx.x == 0) {
         const double N = double(batch->n_tokens);
         batch->trunc_frac = N > 0 ? double(nt) / N : 0.0;
