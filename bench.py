@@ -329,6 +329,8 @@ def run_ours(args):
     end = torch.cuda.Event(enable_timing=True)
     with ClockSampler(dev.index) as clocks:
         torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
         start.record(stream)
         for k in range(args.steps):
             e0, e1, e2, e3 = ev[k]
@@ -350,6 +352,8 @@ def run_ours(args):
             e3.record(stream)
         end.record(stream)
         torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
     total_ms = start.elapsed_time(end)
     if world > 1:
         t = torch.tensor([total_ms], device=dev)
