@@ -107,6 +107,11 @@ SMALL = {
     "ragged_cta": W.small_variant(W.QWEN, name="ragged_cta", n_prompts=2, group_size=3, len_lo=3, len_hi=40,
                                   V=20011, ld_pad=24),
     "qwen_vocab": W.small_variant(W.QWEN, name="qwen_vocab", n_prompts=2, group_size=4, len_lo=8, len_hi=24),
+    # degenerate and wide vocabularies: one token (logp = 0, H = 0, zero gradient), and 2^18 + 3 columns
+    "one_token_vocab": W.small_variant(W.GRPO, name="one_token_vocab", n_prompts=2, group_size=3, len_lo=5,
+                                       len_hi=30, V=1),
+    "wide_vocab": W.small_variant(W.QWEN, name="wide_vocab", n_prompts=2, group_size=2, len_lo=8, len_hi=40,
+                                  V=262147),
 }
 
 
