@@ -4,6 +4,7 @@ element over the whole chain; the full-size workloads on sampled rows plus
 every O(T) output."""
 
 import math
+import os
 
 import numpy as np
 import pytest
@@ -547,3 +548,47 @@ def test_autograd_loss_through_an_lm_head():
     acrl.acrl_loss(step2, logits, b.ids, b.mask, b.logp_mu, b.rewards, b.seq_offsets, b.group_offsets).backward()
     ref = step2.grad.float().t() @ h.float()
     assert torch.allclose(Wt.grad.float(), ref, rtol=2e-2, atol=1e-6 + 2e-2 * float(ref.abs().max()))
+
+
+def _quadrant_rows():
+    path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "acrl_quadrants.txt")
+    with open(path) as f:
+        return [ln.split() for ln in f if ln.strip() and not ln.startswith("#")]
+
+
+def _one_token_controller(pi, mu, A, X, **kw):
+    """One prompt with one response of one token, fed to the O(T) calls as
+    log-probs: Y = D = |pi - mu|, A = R (a singleton prompt), X given."""
+    p = acrl.Params(X_init=X, **kw)
+    f32 = dict(dtype=torch.float32, device=DEV)
+    so = torch.tensor([0, 1], dtype=torch.int64, device=DEV)
+    go = torch.tensor([0, 1], dtype=torch.int32, device=DEV)
+    disc = api.seq_discrepancy(torch.tensor([math.log(pi)], **f32), torch.tensor([math.log(mu)], **f32), None, so, go)
+    adv = api.grpo_advantage(torch.tensor([A], **f32), go, p)
+    w, coef, alpha = api.controller_step(api.controller_init(p), p, disc, None, so, go, adv)
+    return float(w[0]), float(alpha[0]), float(disc.grp_host()[0]["Y"]), p
+
+
+@pytest.mark.parametrize("row", _quadrant_rows(), ids=lambda r: f"{r[0]}-{r[1]}")
+def test_sign_table_on_gpu(row):
+    """Sec. 4.2's eight cases on the GPU: the sign of alpha and whether the
+    weight is above or below 1, for Y > X and Y < X in each (A, pi vs mu)."""
+    regime, _, sA, pvm, salpha, rho_vs = row[:6]
+    pi, mu = (0.3, 0.5) if pvm == "<" else (0.5, 0.3)
+    X = 0.1 if regime == "Y>X" else 0.4                      # Y = |pi - mu| = 0.2
+    w, alpha, Y, p = _one_token_controller(pi, mu, 1.0 if sA == "+" else -1.0, X)
+    assert Y == pytest.approx(0.2, rel=1e-6)
+    assert alpha != 0.0 and (alpha > 0) == (salpha == "+")
+    assert (w > 1.0) == (rho_vs == ">")
+    assert w == pytest.approx(min((pi / mu) ** alpha, p.C), rel=2e-6)
+
+
+def test_controller_special_cases_on_gpu():
+    # Y = X: X set to the Y the GPU computed, so alpha is exactly 0 and the weight exactly 1
+    _, _, Y, _ = _one_token_controller(0.2, 0.4, 1.0, 1.0)
+    w, alpha, _, _ = _one_token_controller(0.2, 0.4, 1.0, Y)
+    assert alpha == 0.0 and w == 1.0
+    w, alpha, _, _ = _one_token_controller(0.2, 0.4, 0.0, 0.013)     # A = 0
+    assert alpha == 0.0 and w == 1.0
+    w, alpha, _, _ = _one_token_controller(0.3, 0.3, 1.0, 0.013)     # mu = pi: rho = 1 for any alpha
+    assert w == 1.0
