@@ -15,14 +15,16 @@
  *     allocates nothing and keeps no global state, except the fixed scratch
  *     array of acrl_lmhead_stats_noalloc (documented there).
  *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL is the
- *     legacy default stream) except acrl_read_flags, which synchronises it.
+ *     legacy default stream) except acrl_read_flags and acrl_check_flags,
+ *     which synchronise it.
  *   - Problems visible on the host (null required pointers, negative sizes,
  *     misalignment, hyper-parameters out of range) return
  *     ACRL_ERR_INVALID_ARG before anything is launched.
  *   - Problems that depend on device data (a sampled id outside [0, V), a
  *     non-finite logit, inconsistent offsets, X <= 0) never trap: the kernel
  *     ORs an ACRL_FLAG_* bit into the caller's device word `dev_flags` and
- *     writes the documented defined value.  acrl_read_flags fetches the word.
+ *     writes the documented defined value.  acrl_read_flags fetches the word;
+ *     acrl_check_flags turns it into a status.
  *   - A failed launch returns ACRL_ERR_CUDA.  Nothing is ever printed.
  *   - bf16 arrays are IEEE bfloat16 bit patterns (acrl_bf16), row-major with a
  *     row stride `ld` in elements; the base pointer must be 16-byte aligned
@@ -51,7 +53,7 @@ typedef enum {
     ACRL_ERR_INVALID_ARG = 1,
     ACRL_ERR_CUDA = 2,
     ACRL_ERR_NOT_IMPLEMENTED = 3,
-    ACRL_ERR_DEVICE_FLAGS = 4,
+    ACRL_ERR_DEVICE_FLAGS = 4,      /* acrl_check_flags: a device flag is set */
     ACRL_ERR_SCRATCH_TOO_SMALL = 5  /* acrl_lmhead_stats_noalloc: the problem needs more
                                        scratch than ACRL_LMHEAD_NOALLOC_SCRATCH_BYTES */
 } acrl_status;
@@ -406,6 +408,11 @@ acrl_status acrl_selftest_wait_timeout(int32_t* dev_flags, int64_t limit_ns, acr
 
 /* Copy the device flags word to *host_flags; synchronises `stream`. */
 acrl_status acrl_read_flags(const int32_t* dev_flags, int32_t* host_flags, acrl_stream stream);
+
+/* Synchronise `stream` and report the device flags word as a status:
+ * ACRL_ERR_DEVICE_FLAGS if any ACRL_FLAG_* bit is set (acrl_read_flags tells
+ * which), ACRL_OK if none.  The word is left as it is. */
+acrl_status acrl_check_flags(const int32_t* dev_flags, acrl_stream stream);
 
 #ifdef __cplusplus
 }

@@ -77,6 +77,7 @@ SIGNATURES = {
     "acrl_lmhead_stats_noalloc": (c_i32, [c_p, c_i64, c_i64, c_i64, c_p, c_i64, c_i64, c_p, c_i64, c_p, c_p, c_p,
                                           c_p, c_p, c_p, c_p]),
     "acrl_read_flags": (c_i32, [c_p, ctypes.POINTER(c_i32), c_p]),
+    "acrl_check_flags": (c_i32, [c_p, c_p]),
     "acrl_selftest_wait_timeout": (c_i32, [c_p, c_i64, c_p]),
 }
 

@@ -318,7 +318,20 @@ def read_flags(flags, stream=None) -> int:
     return int(host.value)
 
 
+def check_flags(flags, stream=None) -> None:
+    """acrl_check_flags: synchronises the stream and raises AcrlError (naming
+    the bits) if any device flag is set."""
+    _need(flags, torch.int32, 1, "flags")
+    dev = _one_device((flags,))
+    with torch.cuda.device(dev):
+        s = torch.cuda.current_stream(dev) if stream is None else stream
+        st = lib().acrl_check_flags(_ptr(flags), s.cuda_stream)
+    if st == _abi.ERR_DEVICE_FLAGS:
+        raise AcrlError(f"device flags raised: 0x{read_flags(flags, stream):x}")
+    check(st, "acrl_check_flags")
+
+
 __all__ = ["Params", "AcrlError", "token_stats", "seq_discrepancy", "grpo_advantage", "controller_init",
-           "controller_step", "loss_grad_logits", "reduce_loss", "read_flags", "read_state", "Discrepancy",
+           "controller_step", "loss_grad_logits", "reduce_loss", "read_flags", "check_flags", "read_state", "Discrepancy",
            "lmhead_logits_stats", "lmhead_merge", "lmhead_workspace_bytes", "save_state", "load_state",
            "struct_buffer", "read_structs", "new_flags", "_abi"]

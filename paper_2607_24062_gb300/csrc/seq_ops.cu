@@ -448,6 +448,13 @@ extern "C" acrl_status acrl_read_flags(const int32_t* dev_flags, int32_t* host_f
     return ACRL_OK;
 }
 
+extern "C" acrl_status acrl_check_flags(const int32_t* dev_flags, acrl_stream stream) {
+    int32_t host = 0;
+    const acrl_status st = acrl_read_flags(dev_flags, &host, stream);
+    if (st != ACRL_OK) return st;
+    return host != 0 ? ACRL_ERR_DEVICE_FLAGS : ACRL_OK;
+}
+
 extern "C" const char* acrl_status_string(acrl_status st) {
     switch (st) {
         case ACRL_OK: return "ok";

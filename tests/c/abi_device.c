@@ -51,7 +51,7 @@ int main(void) {
         fprintf(stderr, "acrl_token_stats failed\n");
         return 1;
     }
-    if (acrl_read_flags(d_flags, &flags, NULL) != ACRL_OK || flags != 0) {
+    if (acrl_check_flags(d_flags, NULL) != ACRL_OK || acrl_read_flags(d_flags, &flags, NULL) != ACRL_OK || flags != 0) {
         fprintf(stderr, "flags %d\n", flags);
         return 1;
     }

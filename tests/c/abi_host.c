@@ -39,6 +39,7 @@ int main(void) {
     CHECK(acrl_loss_grad_logits(NULL, -1, 8, 8, ids, NULL, NULL, NULL, out, NULL, NULL, 0.2f, NULL, out, out, NULL,
                                 NULL) == ACRL_ERR_INVALID_ARG);
     CHECK(acrl_reduce_loss(out, -1, out, NULL) == ACRL_ERR_INVALID_ARG);
+    CHECK(acrl_check_flags(NULL, NULL) == ACRL_ERR_INVALID_ARG);
 
     /* hyper-parameters out of range */
     memset(&p, 0, sizeof p);

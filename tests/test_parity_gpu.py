@@ -314,6 +314,9 @@ def test_bad_ids_nonfinite_and_masked_rows():
     lse, logp, H = api.token_stats(logits, ids, mask, V=V, flags=flags)
     f = api.read_flags(flags)
     assert f == (acrl.FLAG_BAD_ID | acrl.FLAG_NONFINITE)
+    with pytest.raises(acrl.AcrlError, match="device flags raised: 0x3"):
+        api.check_flags(flags)
+    api.check_flags(api.new_flags())     # a clean word is ACRL_OK
     lp = host(logp)
     assert lp[1] == 0.0 and lp[2] == 0.0 and np.isnan(lp[3]) and np.isnan(host(H)[4]) and lp[5] == 0.0
     z = rows_f64(logits, np.arange(T), V)
