@@ -567,6 +567,58 @@ def run_lmhead(args):
     return 0
 
 
+class _PinnedHost:
+    """Page-locked host arrays for the end-to-end run.  First choice: driver
+    allocations of exactly the requested size (cuMemHostAlloc), which move at
+    the link rate whatever the page size.  If that fails: ordinary memory
+    advised onto transparent huge pages before first touch and registered in
+    place (fast only when the kernel finds huge pages for it)."""
+
+    def __init__(self):
+        import ctypes
+        self.ctypes = ctypes
+        self.allocs = []        # cuMemHostAlloc pointers
+        self.registered = []    # registered numpy arrays
+        self.kind = None
+        try:
+            self.cuda = ctypes.CDLL("libcuda.so.1")
+        except OSError:
+            self.cuda = None
+
+    def empty(self, shape, dtype):
+        import torch
+        ct = self.ctypes
+        nbytes = int(np.prod(shape)) * np.dtype(dtype).itemsize
+        if self.cuda is not None and self.kind != "registered":
+            p = ct.c_void_p()
+            if self.cuda.cuMemHostAlloc(ct.byref(p), ct.c_size_t(nbytes), ct.c_uint(0)) == 0 and p.value:
+                self.allocs.append(p)
+                self.kind = "cuMemHostAlloc"
+                buf = (ct.c_uint8 * nbytes).from_address(p.value)
+                return np.frombuffer(buf, dtype=dtype).reshape(shape)
+        if self.kind == "cuMemHostAlloc":
+            raise RuntimeError("cuMemHostAlloc failed for the second buffer")
+        arr = _huge_empty(shape, dtype)
+        if int(torch.cuda.cudart().cudaHostRegister(arr.ctypes.data, arr.nbytes, 0)) != 0:
+            raise RuntimeError("cudaHostRegister failed")
+        self.registered.append(arr)
+        self.kind = "registered"
+        return arr
+
+    def describe(self):
+        return ("user buffers from cuMemHostAlloc (page-locked by the driver)" if self.kind == "cuMemHostAlloc" else
+                "user buffers page-locked in place with cudaHostRegister (advised onto huge pages)")
+
+    def free(self):
+        import torch
+        torch.cuda.synchronize()
+        for p in self.allocs:
+            self.cuda.cuMemFreeHost(p)
+        for arr in self.registered:
+            torch.cuda.cudart().cudaHostUnregister(arr.ctypes.data)
+        self.allocs, self.registered = [], []
+
+
 def _huge_empty(shape, dtype):
     """np.empty whose pages are advised as transparent huge pages (Linux), before any page is touched."""
     import ctypes
@@ -591,21 +643,17 @@ def run_e2e(batch, step, params, args, dev):
     import torch
 
     import paper_2607_24062_gb300 as acrl
-    cudart = torch.cuda.cudart()
     T, ld = batch.logits.shape
     V = batch.V
-    # The user's host arrays, page-locked in place (torch's pinned allocator would round 44.8 GB up to 64 GB).
-    # They are advised onto huge pages before first touch: with 64 KB pages, copies from buffers this large
-    # ran at a fraction of the link rate, with huge pages at the full rate.
-    h_logits_np = _huge_empty((T, ld), np.uint16)
-    h_grad_np = _huge_empty((T, ld), np.uint16)
-    registered = []
+    # The user's host arrays, page-locked and of exactly their size (torch's pinned allocator would round 44.8 GB
+    # up to 64 GB).
+    pinned = _PinnedHost()
     try:
-        for arr in (h_logits_np, h_grad_np):
-            rc = cudart.cudaHostRegister(arr.ctypes.data, arr.nbytes, 0)
-            if int(rc) != 0:
-                return {"value": None, "unit": UNIT, "error": f"cudaHostRegister failed ({int(rc)})"}
-            registered.append(arr)
+        try:
+            h_logits_np = pinned.empty((T, ld), np.uint16)
+            h_grad_np = pinned.empty((T, ld), np.uint16)
+        except RuntimeError as e:
+            return {"value": None, "unit": UNIT, "error": str(e)}
         h_logits = torch.from_numpy(h_logits_np).view(torch.bfloat16)
         h_grad = torch.from_numpy(h_grad_np).view(torch.bfloat16)
         h_logits.copy_(batch.logits)
@@ -694,11 +742,9 @@ def run_e2e(batch, step, params, args, dev):
         return {"value": int(batch.mask.sum()) / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n, "chunks": nchunk,
                 "host_link_GB/s": (h2d + d2h) / (ms / 1e3) / 1e9, "download_matches_device": ok,
-                "host_memory": "user buffers page-locked with cudaHostRegister"}
+                "host_memory": pinned.describe()}
     finally:
-        torch.cuda.synchronize()
-        for arr in registered:
-            cudart.cudaHostUnregister(arr.ctypes.data)
+        pinned.free()
 
 
 def main():
