@@ -82,6 +82,48 @@ def _loss_grad_no_norm(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, se
                                         rows)
 
 
+def _controller_continuous_sign(state, params, *args):
+    """Mistake: the continuous-reduction ablation raises the weight it should lower."""
+    if params.mode == O.MODE_ACRL_CONTINUOUS:
+        params = O.Params(**{**vars(params), "kappa": -params.kappa})
+    return OA._orig["controller_step"](state, params, *args)
+
+
+def _controller_no_moving_average(state, params, *args):
+    """Mistake: the moving-average X never moves."""
+    return OA._orig["controller_step"](state, O.Params(**{**vars(params), "x_ema": 0.0}), *args)
+
+
+def _controller_calibration_by_batch(state, params, lr, mask, so, go, seq, grp, batch, adv):
+    """Mistake: X as the mean of the calibration batches' means instead of over all their prompts."""
+    b2 = dict(batch)
+    b2["Y_sum"] = batch["Y_mean"]
+    b2["n_groups_valid"] = 1 if batch["n_groups_valid"] > 0 else 0
+    return OA._orig["controller_step"](state, params, lr, mask, so, go, seq, grp, b2, adv)
+
+
+def _loss_grad_entropy_sign(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch, params, rows=None):
+    """Mistake: the entropy bonus penalises entropy."""
+    p = O.Params(**{**vars(params), "entropy_coeff": -params.entropy_coeff})
+    return OA._orig["loss_grad_logits"](z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch, p,
+                                        rows)
+
+
+def _discrepancy_token_weighted_Y(logp_pi, logp_mu, mask, so, go, entropy=None):
+    """Mistake: Y_g as the token mean of d over the prompt instead of the mean of its responses' D_i."""
+    lr, d, seq, grp, batch, f = OA._orig["seq_discrepancy"](logp_pi, logp_mu, mask, so, go, entropy)
+    for g in range(len(go) - 1):
+        members = [i for i in range(go[g], go[g + 1]) if seq["n"][i] > 0]
+        ntok = sum(seq["n"][i] for i in members)
+        grp["Y"][g] = sum(seq["mean_d"][i] * seq["n"][i] for i in members) / ntok if ntok else 0.0
+    return lr, d, seq, grp, batch, f
+
+
+def _lmhead_not_rounded(hidden, weight):
+    """Mistake: the logits kept at full precision instead of the engine's bf16."""
+    return np.asarray(hidden, dtype=np.float64) @ np.asarray(weight, dtype=np.float64).T
+
+
 def _round_bf16_truncates(x):
     x = np.asarray(x, dtype=np.float64)
     f, e = np.frexp(x)
@@ -96,10 +138,14 @@ PIN_GROUPS = {
     "grpo_advantage": [lambda: P.test_grpo_binary_closed_form(8, 3), P.test_grpo_matches_scipy_zscore,
                        P.test_grpo_special_groups],
     "controller_step": [lambda: [P.test_quadrant_sign_table(r) for r in P._read_quadrants()],
-                        P.test_controller_special_cases, P.test_tis_and_mis_thresholds],
+                        P.test_controller_special_cases, P.test_tis_and_mis_thresholds,
+                        lambda: [P.test_continuous_reduction_always_reduces(r) for r in P._read_quadrants()],
+                        P.test_continuous_reduction_kappa, P.test_moving_average_X_by_hand,
+                        P.test_calibration_averages_prompts_across_batches],
     "loss_grad_logits": [lambda: P.test_gradient_matches_autograd(False, 0.0), P.test_on_policy_loss_by_hand_and_invariants,
-                         lambda: P.test_gradient_central_differences(0.0)],
+                         lambda: P.test_gradient_central_differences(0.0), P.test_entropy_bonus_by_hand],
     "round_bf16": [P.test_round_bf16_matches_library_and_ties],
+    "lmhead_logits": [P.test_lmhead_logits_small],
 }
 
 MUTATIONS = [
@@ -114,6 +160,12 @@ MUTATIONS = [
     ("loss_grad_logits", "one-hot at the wrong column", _loss_grad_wrong_column),
     ("loss_grad_logits", "prompt count left out of the normalisation", _loss_grad_no_norm),
     ("round_bf16", "truncation instead of round-to-nearest-even", _round_bf16_truncates),
+    ("controller_step", "continuous reduction with the opposite sign", _controller_continuous_sign),
+    ("controller_step", "moving-average X never applied", _controller_no_moving_average),
+    ("controller_step", "X from the mean of batch means", _controller_calibration_by_batch),
+    ("loss_grad_logits", "entropy bonus with the wrong sign", _loss_grad_entropy_sign),
+    ("seq_discrepancy", "Y_g weighted by tokens instead of responses", _discrepancy_token_weighted_Y),
+    ("lmhead_logits", "logits not rounded to bf16", _lmhead_not_rounded),
 ]
 
 

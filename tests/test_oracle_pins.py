@@ -321,6 +321,22 @@ def test_multi_step_calibration():
     assert st.calibrated and st.X == pytest.approx(0.02, abs=1e-15)
 
 
+def test_calibration_averages_prompts_across_batches():
+    # X is the mean of Y_g over every prompt of the calibration batches (Sec. 4.1): batches of 1 and 3 prompts
+    # give (0.01 + 3 x 0.03) / 4 = 0.025, not the mean of the two batch means (0.02)
+    p = O.Params(calib_steps=2)
+    st = O.controller_init(p)
+    for Ys in ([0.01], [0.03, 0.03, 0.03]):
+        G = len(Ys)
+        lr = np.full(G, 0.5)
+        seq = {"n": np.ones(G, dtype=np.int64), "group": np.arange(G), "mean_d": np.array(Ys), "sum_lr": lr}
+        grp = {"Y": np.array(Ys), "n_valid_seqs": np.ones(G, dtype=np.int64)}
+        batch = {"Y_sum": sum(Ys), "Y_mean": sum(Ys) / G, "n_groups_valid": G}
+        offs = list(range(G + 1))
+        _, _, st, _, _ = O.controller_step(st, p, lr, None, offs, offs, seq, grp, batch, np.ones(G))
+    assert st.calibrated and st.X == pytest.approx(0.025, abs=1e-15)
+
+
 def test_nonpositive_X_flag_and_fixed_point():
     # mu = pi everywhere: d = 0, X calibrates to 0, alpha := 0 and every weight is 1
     rng = np.random.default_rng(2)
