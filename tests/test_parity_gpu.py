@@ -595,3 +595,31 @@ def test_controller_special_cases_on_gpu():
     assert alpha == 0.0 and w == 1.0
     w, alpha, _, _ = _one_token_controller(0.3, 0.3, 1.0, 0.013)     # mu = pi: rho = 1 for any alpha
     assert w == 1.0
+
+
+def test_calibration_over_prompts_of_two_batches_on_gpu():
+    """calib_steps = 2 over batches of 1 and 3 prompts: X is the mean of Y_g
+    over all four prompts (Sec. 4.1), not the mean of the two batch means."""
+    p = acrl.Params(calib_steps=2)
+    op = oracle_params(p)
+    state, ost = api.controller_init(p), O.controller_init(op)
+    f32 = dict(dtype=torch.float32, device=DEV)
+    Ys = []
+    for G, mu in ((1, 0.31), (3, 0.36)):
+        lp_pi = torch.full((G,), math.log(0.3), **f32)
+        lp_mu = torch.full((G,), math.log(mu), **f32)
+        so = torch.arange(G + 1, dtype=torch.int64, device=DEV)
+        go = torch.arange(G + 1, dtype=torch.int32, device=DEV)
+        disc = api.seq_discrepancy(lp_pi, lp_mu, None, so, go)
+        adv = api.grpo_advantage(torch.ones(G, **f32), go, p)
+        api.controller_step(state, p, disc, None, so, go, adv)
+        lr, d, seq, grp, batch, _ = O.seq_discrepancy(host(lp_pi).astype(np.float64), host(lp_mu).astype(np.float64),
+                                                      None, host(so), host(go))
+        ost = O.controller_step(ost, op, lr, None, host(so), host(go), seq, grp, batch, np.ones(G))[2]
+        Ys.append(list(disc.grp_host()["Y"]))
+    st = api.read_state(state)
+    assert bool(st["calibrated"]) and ost.calibrated
+    assert_close_rel(float(st["X"]), ost.X, floor=1e-12, what="X")
+    by_prompt = (sum(Ys[0]) + sum(Ys[1])) / 4
+    assert float(st["X"]) == pytest.approx(by_prompt, rel=1e-12)
+    assert abs(by_prompt - (np.mean(Ys[0]) + np.mean(Ys[1])) / 2) > 1e-3 * by_prompt
