@@ -72,9 +72,9 @@ typedef enum {
     ACRL_MODE_TIS = 1,    /* token-level truncated IS (Eq. TIS): min(pi/mu, C)  */
     ACRL_MODE_MIS = 2,    /* sequence-level masked IS (Eq. MIS): rho_i 1{rho_i<=C} */
     ACRL_MODE_ACRL = 3,   /* Eq. ACRL: min((pi/mu)^alpha, C)                    */
-    ACRL_MODE_ACRL_CONTINUOUS = 4, /* Sec. 5.5 ablation "continuous reduction":
+    ACRL_MODE_ACRL_CONTINUOUS = 4, /* Sec. 5.5 ablation, continuous reduction:
                                       alpha = -kappa sign(A), no Y/X comparison   */
-    ACRL_MODE_ACRL_FALLBACK = 5    /* Sec. 5.5 ablation "fallback to GRPO": the ACRL
+    ACRL_MODE_ACRL_FALLBACK = 5    /* Sec. 5.5 ablation, fallback to GRPO: the ACRL
                                       alpha when Y > X, alpha = 0 (w = 1) otherwise */
 } acrl_mode;
 
@@ -82,7 +82,7 @@ typedef enum {
 typedef enum {
     ACRL_Y_GROUP = 0,     /* Y_g = (1/G) sum_i D_i over the prompt's responses (the formula) */
     ACRL_Y_SEQUENCE = 1,  /* Y = D_i, the response's own mean distance                       */
-    ACRL_Y_BATCH = 2      /* Y = mean over prompts of Y_g (the "step discrepancy")            */
+    ACRL_Y_BATCH = 2      /* Y = mean over prompts of Y_g (the step discrepancy)            */
 } acrl_y_granularity;
 
 typedef enum {
@@ -248,7 +248,7 @@ acrl_status acrl_controller_init(acrl_controller_state* state, const acrl_params
 
 /*
  * acrl_controller_step -- the adaptive controller and the importance weights.
- * Calibration (Sec. 4.1, X "compiled before training"; Sec. 5.1 takes it from
+ * Calibration (Sec. 4.1, X fixed before training; Sec. 5.1 takes it from
  * step 0): while not calibrated, Y_sum and Q_eff of `batch` are added to the
  * state; after p->calib_steps batches X = sum / count is frozen.  On earlier
  * calibration batches alpha = 0.  Then per response (Sec. 4.1, after Eq. ACRL)

@@ -26,7 +26,7 @@ readings of the CUDA path; each is listed with its reason in the design notes):
   * min(rho, C) is evaluated as exp(min(alpha*lr, ln C)); the MIS indicator
     1{rho_i <= C} as S_i <= ln C.
   * X is the mean of Y_g over the prompts of the first `calib_steps` batches
-    (Sec. 4.1, "compiled before training"; Sec. 5.1 takes it from step 0), then
+    (Sec. 4.1: fixed before training; Sec. 5.1 takes it from step 0), then
     frozen.  If X <= 0 the controller sets alpha = 0 and raises a flag.
   * The clip tie r = 1 +/- eps keeps the unclipped branch.
   * Masked tokens contribute nothing: their outputs are 0 and their gradient
