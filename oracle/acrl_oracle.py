@@ -312,7 +312,9 @@ def grpo_advantage(rewards, group_offsets, params: Params):
             continue
         mean = r.sum() / G
         var = ((r - mean) ** 2).sum() / (G - params.adv_ddof) if G > params.adv_ddof else 0.0
-        A[go[g]:go[g + 1]] = (r - mean) / (math.sqrt(var) + params.adv_eps)
+        den = math.sqrt(var) + params.adv_eps
+        # equal rewards with adv_eps = 0 give 0/0: such a prompt carries no advantage, A = 0
+        A[go[g]:go[g + 1]] = (r - mean) / den if den > 0 else 0.0
     return A
 
 

@@ -202,6 +202,13 @@ def test_grpo_matches_scipy_zscore():
                                        rtol=1e-12)
 
 
+def test_grpo_equal_rewards_without_epsilon():
+    # all-equal rewards with adv_eps = 0: the definition's 0/0 is read as no advantage
+    A = O.grpo_advantage(np.array([1.0, 1.0, 1.0, 0.0, 1.0]), [0, 3, 5], O.Params(adv_eps=0.0))
+    assert np.all(A[:3] == 0.0)
+    np.testing.assert_allclose(A[3:], [-math.sqrt(0.5), math.sqrt(0.5)], rtol=1e-14)   # (0 or 1 - 0.5) / sqrt(0.5)
+
+
 def test_grpo_special_groups():
     R = np.array([0.7, 1.0, 1.0, 1.0, 0.0])
     A = O.grpo_advantage(R, [0, 1, 4, 4, 5], O.Params())

@@ -151,7 +151,7 @@ def test_modes(mode, y_gran):
     _full_chain_check(_gen(spec, seed=77), acrl.Params(mode=mode, y_gran=y_gran, gamma=1.3, C=5.0))
 
 
-@pytest.mark.parametrize("kw", [dict(agg=acrl.AGG_TOKEN_MEAN), dict(adv_ddof=0), dict(X_init=0.013),
+@pytest.mark.parametrize("kw", [dict(agg=acrl.AGG_TOKEN_MEAN), dict(adv_ddof=0), dict(adv_eps=0.0), dict(X_init=0.013),
                                 dict(singleton_rule=acrl.SINGLETON_ZERO), dict(calib_steps=2),
                                 dict(entropy_coeff=0.001), dict(entropy_coeff=0.05, agg=acrl.AGG_TOKEN_MEAN),
                                 dict(X_init=0.013, x_ema=0.3), dict(mode=acrl.MODE_ACRL_CONTINUOUS, kappa=3.0)])
