@@ -238,8 +238,11 @@ def seq_discrepancy(logp_pi, logp_mu, mask, seq_offsets, group_offsets, entropy=
     flags = 0 if ok else FLAG_BAD_OFFSETS
     S, Gn = len(so) - 1, len(go) - 1
 
-    lr = np.where(m, pi - mu, 0.0)
+    with np.errstate(invalid="ignore"):
+        lr = np.where(m, pi - mu, 0.0)
     d = np.where(m, np.abs(np.exp(pi) - np.exp(mu)), 0.0)
+    if np.any(np.isnan(lr[m])):
+        flags |= FLAG_NONFINITE         # a NaN log-prob on either side of a valid token
     Hm = None if entropy is None else np.where(m, np.asarray(entropy, dtype=np.float64), 0.0)
 
     seq = {k: np.zeros(S) for k in ("mean_d", "max_d", "sum_d", "sum_d2", "sum_lr", "mean_H")}
@@ -390,11 +393,12 @@ def controller_step(state: ControllerState, params: Params, lr, mask, seq_offset
                 w[t] = 1.0
             elif params.mode == MODE_MIS:
                 S_i = seq["sum_lr"][i]
-                w[t] = math.exp(S_i) if S_i <= logC else 0.0
+                w[t] = math.exp(S_i) if S_i <= logC else 0.0     # a NaN S_i fails the test: weight 0
                 n_trunc += S_i > logC
             else:
-                log_rho = alpha[i] * lr[t]
-                w[t] = math.exp(min(log_rho, logC))
+                # rho^0 = 1 even where the log-ratio is infinite (mu = 0); a NaN log-ratio gets weight 0
+                log_rho = 0.0 if alpha[i] == 0.0 else alpha[i] * lr[t]
+                w[t] = 0.0 if math.isnan(log_rho) else math.exp(min(log_rho, logC))
                 n_trunc += log_rho > logC
     N = int(m.sum())
     valid_seq = np.asarray(seq["n"]) > 0

@@ -56,12 +56,14 @@ __global__ void __launch_bounds__(kSeqThreads) seq_stats_kernel(
     int n = 0;
     double sd = 0.0, sd2 = 0.0, slr = 0.0, sH = 0.0;
     float mxd = 0.f;
+    bool nan_lr = false;
     for (int64_t t = lo + threadIdx.x; t < hi; t += kSeqThreads) {
         const bool m = mask ? mask[t] != 0 : true;
         float l = 0.f, dd = 0.f;
         if (m) {
             const float a = logp_pi[t], b = logp_mu[t];
             l = a - b;
+            nan_lr |= isnan(l);  // a NaN log-prob on either side
             dd = prob_distance(a, b);
             ++n;
             sd += dd;
@@ -73,6 +75,7 @@ __global__ void __launch_bounds__(kSeqThreads) seq_stats_kernel(
         lr[t] = l;
         d[t] = dd;
     }
+    if (nan_lr) raise_flag(flags, ACRL_FLAG_NONFINITE);
     double v[5] = {double(n), sd, sd2, slr, sH}, mx = mxd;
     block_sums_max0<NW, 5>(v, mx, sh);
     n = int(v[0]);
@@ -322,7 +325,7 @@ __global__ void __launch_bounds__(kSeqThreads) controller_weights_kernel(
     const float escale = norm > 0.0 ? float(double(p.entropy_coeff) / norm) : 0.f;
     const float Si = float(s.sum_lr);
     const bool mis_cut = Si > logC;
-    const float w_mis = mis_cut ? 0.f : expf(Si);
+    const float w_mis = (mis_cut || isnan(Si)) ? 0.f : expf(Si);
     int nt = 0;
     double sw = 0.0;
     for (int64_t t = lo + threadIdx.x; t < hi; t += kSeqThreads) {
@@ -335,8 +338,9 @@ __global__ void __launch_bounds__(kSeqThreads) controller_weights_kernel(
                 w = w_mis;
                 nt += mis_cut;
             } else {
-                const float lrho = s.alpha * lr[t];
-                w = expf(fminf(lrho, logC));
+                // rho^0 = 1 even where the log-ratio is infinite (mu = 0); a NaN log-ratio gets weight 0
+                const float lrho = s.alpha == 0.f ? 0.f : s.alpha * lr[t];
+                w = isnan(lrho) ? 0.f : expf(fminf(lrho, logC));
                 nt += lrho > logC;
             }
             sw += w;

@@ -328,6 +328,32 @@ def test_multi_step_calibration():
     assert st.calibrated and st.X == pytest.approx(0.02, abs=1e-15)
 
 
+def _lr_case(lr_value, A, mode=O.MODE_ACRL, Y=0.026, X=0.013):
+    lr = np.array([lr_value])
+    seq = {"n": np.array([1]), "group": np.array([0]), "mean_d": np.array([Y]), "sum_lr": lr.copy()}
+    grp = {"Y": np.array([Y]), "n_valid_seqs": np.array([1])}
+    batch = {"Y_sum": Y, "Y_mean": Y, "n_groups_valid": 1}
+    p = O.Params(mode=mode, X_init=X)
+    return O.controller_step(O.controller_init(p), p, lr, None, [0, 1], [0, 1], seq, grp, batch, np.array([A]))
+
+
+def test_infinite_and_nan_log_ratios():
+    # mu = 0 on a sampled token: lr = +inf.  rho^0 = 1 (A = 0 gives alpha = 0), TIS truncates at C, an
+    # exponent of either sign follows min(rho^alpha, C) (C, or 0); MIS truncates the sequence
+    assert _lr_case(math.inf, 0.0)[0][0] == 1.0
+    assert _lr_case(math.inf, 1.0, mode=O.MODE_TIS)[0][0] == pytest.approx(3.0, rel=1e-15)
+    assert _lr_case(math.inf, -1.0)[0][0] == pytest.approx(3.0, rel=1e-15)  # Y > X, A < 0: alpha > 0
+    assert _lr_case(math.inf, 1.0)[0][0] == 0.0           # Y > X, A > 0: alpha < 0
+    assert _lr_case(math.inf, 1.0, mode=O.MODE_MIS)[0][0] == 0.0
+    # a NaN log-prob: the token's weight is 0 and the discrepancy pass flags it
+    for mode in (O.MODE_ACRL, O.MODE_TIS, O.MODE_MIS):
+        assert _lr_case(math.nan, 1.0, mode=mode)[0][0] == 0.0
+    *_, f = O.seq_discrepancy(np.array([-1.0, -2.0]), np.array([-1.5, math.nan]), None, [0, 2], [0, 1])
+    assert f & O.FLAG_NONFINITE
+    lr, d, *_, f = O.seq_discrepancy(np.array([-1.0]), np.array([-math.inf]), None, [0, 1], [0, 1])
+    assert f == 0 and lr[0] == math.inf and d[0] == pytest.approx(math.exp(-1.0), rel=1e-15)
+
+
 def test_calibration_averages_prompts_across_batches():
     # X is the mean of Y_g over every prompt of the calibration batches (Sec. 4.1): batches of 1 and 3 prompts
     # give (0.01 + 3 x 0.03) / 4 = 0.025, not the mean of the two batch means (0.02)

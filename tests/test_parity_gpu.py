@@ -623,3 +623,28 @@ def test_calibration_over_prompts_of_two_batches_on_gpu():
     by_prompt = (sum(Ys[0]) + sum(Ys[1])) / 4
     assert float(st["X"]) == pytest.approx(by_prompt, rel=1e-12)
     assert abs(by_prompt - (np.mean(Ys[0]) + np.mean(Ys[1])) / 2) > 1e-3 * by_prompt
+
+
+def test_infinite_and_nan_rollout_log_probs_on_gpu():
+    """mu = 0 on a sampled token (log mu = -inf) and a NaN log-prob, fed to
+    the O(T) calls: the weights and flags the oracle gives."""
+    f32 = dict(dtype=torch.float32, device=DEV)
+    so = torch.tensor([0, 1, 2, 3], dtype=torch.int64, device=DEV)
+    go = torch.tensor([0, 1, 2, 3], dtype=torch.int32, device=DEV)
+    lp_pi = torch.tensor([-1.0, -1.0, -1.0], **f32)
+    lp_mu = torch.tensor([-math.inf, -math.inf, math.nan], **f32)
+    for mode, A in ((acrl.MODE_ACRL, (0.0, 1.0, -1.0)), (acrl.MODE_TIS, (1.0, 1.0, 1.0)),
+                    (acrl.MODE_MIS, (1.0, -1.0, 1.0))):
+        p = acrl.Params(mode=mode, X_init=0.1)
+        op = oracle_params(p)
+        flags = api.new_flags()
+        disc = api.seq_discrepancy(lp_pi, lp_mu, None, so, go, flags=flags)
+        adv = torch.tensor(A, **f32)
+        w, coef, alpha = api.controller_step(api.controller_init(p), p, disc, None, so, go, adv, flags=flags)
+        lr, d, seq, grp, batch, of = O.seq_discrepancy(host(lp_pi).astype(np.float64), host(lp_mu).astype(np.float64),
+                                                       None, host(so), host(go))
+        ow, oalpha, *_ = O.controller_step(O.controller_init(op), op, lr, None, host(so), host(go), seq, grp, batch,
+                                           np.array(A))
+        assert api.read_flags(flags) & acrl.FLAG_NONFINITE and of & O.FLAG_NONFINITE
+        np.testing.assert_allclose(host(w), ow, rtol=1e-6, atol=0, err_msg=f"mode {mode}")
+        assert host(w)[2] == 0.0
