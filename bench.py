@@ -518,20 +518,22 @@ def run_lmhead(args):
         if ev:
             ev[1].record(stream)
         acrl.api.lmhead_merge(partials, logits, b.ids, b.mask, N=N, lse=lse, logp=logp, entropy=ent, flags=flags)
+        if ev:
+            ev[2].record(stream)
         disc = acrl.seq_discrepancy(logp, b.logp_mu, b.mask, b.seq_offsets, b.group_offsets, ent, flags=flags)
         adv = acrl.grpo_advantage(b.rewards, b.group_offsets, p, flags=flags)
         w, coef, alpha = acrl.controller_step(state, p, disc, b.mask, b.seq_offsets, b.group_offsets, adv,
                                               flags=flags)
         if ev:
-            ev[2].record(stream)
+            ev[3].record(stream)
         acrl.loss_grad_logits(logits, b.ids, b.mask, lse, None, coef, p.clip_eps, V=N, grad=grad, flags=flags)
         if ev:
-            ev[3].record(stream)
+            ev[4].record(stream)
 
     for _ in range(args.warmup):
         one()
     torch.cuda.synchronize()
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(dev.index) as clocks:
         torch.cuda.synchronize()
@@ -543,7 +545,8 @@ def run_lmhead(args):
     fl = acrl.read_flags(flags)
     total_ms = t0.elapsed_time(t1)
     gemm_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in evs]))
-    grad_ms = float(np.mean([e[2].elapsed_time(e[3]) for e in evs]))
+    merge_ms = float(np.mean([e[1].elapsed_time(e[2]) for e in evs]))
+    grad_ms = float(np.mean([e[3].elapsed_time(e[4]) for e in evs]))
     flop = 2.0 * M * N * K
     tf = flop / (gemm_ms / 1e3) / 1e12
     peak, kind = _peak_tflops()
@@ -557,6 +560,7 @@ def run_lmhead(args):
                         "unit": "TFLOP/s", "frac": tf / peak, "traffic": None, "peak_kind": kind,
                         "flop_per_launch": flop, "ms_per_launch": gemm_ms},
            "kernels": {"acrl_lmhead_logits_stats": {"ms": gemm_ms, "TFLOP/s": tf},
+                       "acrl_lmhead_merge": {"ms": merge_ms},
                        "acrl_loss_grad_logits": {"ms": grad_ms,
                                                  "GB/s": 4.0 * M * N / (grad_ms / 1e3) / 1e9}},
            "clocks": clocks.summary(), "gpu_launches": 10 * args.steps}

@@ -446,26 +446,47 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
 }
 
-// Merge of the per-tile states of each row: lse, logp and entropy.  One
-// thread per row, tiles in order (deterministic); partials are [n_tiles][M].
+// Merge of the per-tile states of each row: lse, logp and entropy.  Eight
+// lanes per row, lane j folding tiles j, j+8, ... in order, then a fixed
+// butterfly over the eight (deterministic); partials are [n_tiles][M].
+constexpr int kMergeLanes = 8;
+
 __global__ void lmhead_merge_kernel(const float4* __restrict__ partials, const acrl_bf16* __restrict__ logits, int M,
                                     int N, int64_t ldl, int n_tiles, const int32_t* __restrict__ ids,
                                     const uint8_t* __restrict__ mask, float* __restrict__ lse, float* __restrict__ logp,
                                     float* __restrict__ ent, int32_t* flags) {
-    const int row = blockIdx.x * blockDim.x + threadIdx.x;
-    if (row >= M) return;
+    const int64_t g = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    const int row = int(g / kMergeLanes), sub = int(g % kMergeLanes);
+    if (row >= M) return;  // the row's eight lanes leave together
     if (mask && mask[row] == 0) {
-        lse[row] = logp[row] = ent[row] = 0.f;
+        if (sub == 0) lse[row] = logp[row] = ent[row] = 0.f;
         return;
     }
     LseAcc acc = lse_empty();
     float mx = -INFINITY;
-    for (int n = 0; n < n_tiles; ++n) {
+    for (int n = sub; n < n_tiles; n += kMergeLanes) {
         const float4 p = partials[int64_t(n) * M + row];
         acc = lse_merge(acc, LseAcc{p.y, p.z, p.w});
         mx = fmaxf(mx, p.x);
     }
-    row_outputs(acc, mx, logits + int64_t(row) * ldl, N, ids[row], lse, logp, ent, row, flags);
+    const unsigned group = 0xffu << (threadIdx.x & 31 & ~(kMergeLanes - 1));
+#pragma unroll
+    for (int m = kMergeLanes / 2; m >= 1; m >>= 1) {
+        const LseAcc o{__shfl_xor_sync(group, acc.U, m), __shfl_xor_sync(group, acc.s0, m),
+                       __shfl_xor_sync(group, acc.s1, m)};
+        acc = lse_merge(acc, o);
+        mx = fmaxf(mx, __shfl_xor_sync(group, mx, m));
+    }
+    if (sub == 0) row_outputs(acc, mx, logits + int64_t(row) * ldl, N, ids[row], lse, logp, ent, row, flags);
+}
+
+acrl_status launch_merge(const float4* partials, const acrl_bf16* logits, int64_t M, int64_t N, int64_t ldl,
+                         const int32_t* ids, const uint8_t* mask, float* lse, float* logp, float* entropy,
+                         int32_t* flags, cudaStream_t s) {
+    const int threads = 256, rows_per_block = threads / kMergeLanes;
+    lmhead_merge_kernel<<<unsigned((M + rows_per_block - 1) / rows_per_block), threads, 0, s>>>(
+        partials, logits, int(M), int(N), ldl, int((N + kBN - 1) / kBN), ids, mask, lse, logp, entropy, flags);
+    return launch_status();
 }
 
 bool encode_map(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows,
@@ -549,11 +570,8 @@ extern "C" acrl_status acrl_lmhead_merge(const float* partials, const acrl_bf16*
     if (M == 0) return ACRL_OK;
     if (!partials || !logits || !ids || !lse || !logp || !entropy) return ACRL_ERR_INVALID_ARG;
     if (!aligned16(partials)) return ACRL_ERR_INVALID_ARG;
-    const int threads = 128;
-    lmhead_merge_kernel<<<unsigned((M + threads - 1) / threads), threads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-        reinterpret_cast<const float4*>(partials), logits, int(M), int(N), ldl, int((N + kBN - 1) / kBN), ids, mask,
-        lse, logp, entropy, dev_flags);
-    return launch_status();
+    return launch_merge(reinterpret_cast<const float4*>(partials), logits, M, N, ldl, ids, mask, lse, logp, entropy,
+                        dev_flags, reinterpret_cast<cudaStream_t>(stream));
 }
 
 // ---------------------------------------------------------------------------
@@ -613,9 +631,6 @@ extern "C" acrl_status acrl_lmhead_stats_noalloc(const acrl_bf16* hidden, int64_
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     const acrl_status st = launch_lmhead<LmRing>(hidden, M, K, ldh, weight, N, ldw, logits, ldl, partials, dev_flags, s);
     if (st != ACRL_OK) return st;
-    const int threads = 128;
-    lmhead_merge_kernel<<<unsigned((M + threads - 1) / threads), threads, 0, s>>>(
-        partials, logits, int(M), int(N), ldl, int((N + kBN - 1) / kBN), ids, mask, lse, logp, entropy, dev_flags);
-    return launch_status();
+    return launch_merge(partials, logits, M, N, ldl, ids, mask, lse, logp, entropy, dev_flags, s);
 }
 
