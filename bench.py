@@ -389,6 +389,7 @@ def run_ours(args):
         return float(np.median([a.elapsed_time(b) for a, b in evs]))
 
     co_ms = median_ms(cached_old, min(5, args.steps))
+    weights_sec54 = _weight_calls_ms(acrl, W, dev, median_ms) if rank == 0 else None
     eb_ms = median_ms(entropy_bonus, min(5, args.steps))
     live_e = mask_h & (ids_h >= 0) & (ids_h < batch.V)
     eb_bytes = int(live_e.sum()) * 4 * V + (batch.T - int(live_e.sum())) * 2 * V + batch.T * 25
@@ -458,6 +459,7 @@ def run_ours(args):
             "acrl_loss_grad_logits (entropy bonus)": {
                 "ms": eb_ms, "GB/s": eb_bytes / (eb_ms / 1e3) / 1e9, "frac": eb_bytes / (eb_ms / 1e3) / 1e9 / peak,
                 "bytes": eb_bytes},
+            "weight calls on the Sec. 5.4 batch shape": weights_sec54,
             "whole_step_GB/s": (k1_bytes + k5_bytes) / (ms_per_step / 1e3) / 1e9,
             "step_replayed_from_cuda_graph": ({"ms": graph_ms, "tokens/s": n_valid / (graph_ms / 1e3)}
                                               if graph_ms else None),
@@ -472,6 +474,30 @@ def run_ours(args):
         out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
     print(json.dumps(out))
     return 0
+
+
+def _weight_calls_ms(acrl, W, dev, median_ms):
+    """The three calls that make the importance weights from per-token
+    log-probs (seq_discrepancy, grpo_advantage, controller_step) on a batch of
+    the shape of the paper's overhead measurement (64 prompts x 8 responses,
+    lengths U[1, 2048]); the paper reports 0.059 s for its call on that
+    setting, hardware not stated."""
+    spec = W.WEIGHTS_SEC54
+    d = W.token_level(spec, W.seed_for(spec.name), device=dev)
+    p = acrl.Params()
+    state = acrl.controller_init(p, device=dev)
+    flags = acrl.api.new_flags(dev)
+
+    def calls():
+        disc = acrl.seq_discrepancy(d["logp_pi"], d["logp_mu"], d["mask"], d["seq_offsets"], d["group_offsets"],
+                                    flags=flags)
+        adv = acrl.grpo_advantage(d["rewards"], d["group_offsets"], p, flags=flags)
+        acrl.controller_step(state, p, disc, d["mask"], d["seq_offsets"], d["group_offsets"], adv, flags=flags)
+
+    ms = median_ms(calls, 20)
+    return {"ms": ms, "tokens": int(d["mask"].sum()), "rows": d["T"], "flags": acrl.read_flags(flags),
+            "workload": W.describe(spec) + ", token-level log-probs only",
+            "note": "includes the output allocations of the Python calls; the paper's 0.059 s is context only"}
 
 
 def _peak_tflops():

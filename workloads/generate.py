@@ -75,6 +75,12 @@ LONG = WorkloadSpec("long", 8, 4, 4096, 16384, 151936, dist="normal", scale=2.0,
 # profiler capture, still far larger than L2.
 QWEN_PROFILE = replace(QWEN, name="qwen_profile", n_prompts=2, group_size=4, len_lo=1024, len_hi=1024)
 
+# The batch of the paper's overhead measurement (Sec. 5.4 on the App. A 3B
+# setting: 64 prompts x 8 responses, responses up to 2048 tokens), for the
+# weight calls alone (token-level inputs, no logits).
+WEIGHTS_SEC54 = WorkloadSpec("weights_sec54", 64, 8, 1, 2048, 151936, reward_p=0.3, perturb_frac=0.1,
+                             perturb_std=0.3)
+
 SPECS = {s.name: s for s in (TINY, GRPO, QWEN, LONG, QWEN_PROFILE)}
 BASE_SEED = 2607_24062
 
@@ -376,7 +382,7 @@ def describe(spec: WorkloadSpec) -> str:
             f"V={spec.V} ld={spec.ld} {spec.dist}(scale={spec.scale}) fp8={spec.fp8_scale}/{spec.fp8_round}")
 
 
-__all__ = ["WorkloadSpec", "TINY", "GRPO", "QWEN", "LONG", "LMHEAD", "SPECS", "generate", "make_structure",
+__all__ = ["WorkloadSpec", "TINY", "GRPO", "QWEN", "LONG", "LMHEAD", "WEIGHTS_SEC54", "SPECS", "generate", "make_structure",
            "generate_lmhead", "LMHeadBatch", "LMHEAD_K", "LMHEAD_W_STD",
            "e4m3_roundtrip", "e4m3_values", "seed_for", "small_variant", "token_level", "Batch",
            "expected_tokens", "describe", "E4M3_MAX"]
