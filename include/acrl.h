@@ -29,6 +29,9 @@
  *   - bf16 arrays are IEEE bfloat16 bit patterns (acrl_bf16), row-major with a
  *     row stride `ld` in elements; the base pointer must be 16-byte aligned
  *     and ld a multiple of 8, so every row starts on a 16-byte boundary.
+ *   - Sizes: 1 <= V <= 2^30 (column indices stay in 32-bit range); the row
+ *     count T is 64-bit (T * ld may exceed 2^32).  Larger V is
+ *     ACRL_ERR_INVALID_ARG.
  *
  * Notation: T token rows, V vocabulary size, S responses (sequences),
  * Gn prompts (groups), m_t in {0,1} the response mask, a_t the sampled id.

@@ -48,6 +48,11 @@ def test_host_side_rejections(L):
     assert L.acrl_token_stats(fake + 2, 4, 16, 16, fake, None, fake, fake, fake, fake, None) == E
     assert L.acrl_token_stats(fake, 4, 16, 16, fake, None, None, fake, fake, fake, None) == E
     assert L.acrl_token_stats(fake, -1, 16, 16, fake, None, fake, fake, fake, fake, None) == E
+    # V above 2^30 (column indices must stay in 32-bit range), for every vocabulary-wide call
+    big = (1 << 30) + 8
+    assert L.acrl_token_stats(fake, 4, big, big, fake, None, fake, fake, fake, fake, None) == E
+    assert L.acrl_loss_grad_logits(fake, 4, big, big, fake, None, fake, None, fake, None, None, 0.2, fake, fake, fake,
+                                   fake, None) == E
     # T = 0 is a valid no-op
     assert L.acrl_token_stats(None, 0, 16, 16, None, None, None, None, None, None, None) == _abi.OK
     # hyper-parameters out of range
