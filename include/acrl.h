@@ -223,7 +223,10 @@ acrl_status acrl_token_stats(const acrl_bf16* logits, int64_t T, int64_t V, int6
  *   seq [S], grp [Gn], batch [1]  device outputs (the controller fields of
  *             seq and batch are written later by acrl_controller_step).
  * Offsets that break the rules above raise BAD_OFFSETS; the offending
- * response is treated as empty.  Deterministic: fixed reduction order, fp64
+ * response is treated as empty, and rows that no well-formed response covers
+ * are not written (here, nor by acrl_controller_step): their lr, d, weight
+ * and coef keep whatever the buffers held, so a caller that sees the flag
+ * must discard the step.  Deterministic: fixed reduction order, fp64
  * accumulation.
  */
 acrl_status acrl_seq_discrepancy(const float* logp_pi, const float* logp_mu, const uint8_t* mask,
