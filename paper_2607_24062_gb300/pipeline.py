@@ -110,7 +110,11 @@ class AcrlStep:
         """Record one whole step over `batch`'s buffers as a CUDA graph (the
         kernels' launches only; no host work is left in the step).  Returns the
         torch.cuda.CUDAGraph; `graph.replay()` runs the step again on whatever
-        the buffers then hold.  `exchange` must be capturable (e.g. NCCL)."""
+        the buffers then hold.  `exchange` must be capturable (e.g. NCCL).
+        Capturing runs the step once eagerly first, so it advances the
+        controller like any step (it calibrates X on `batch` if X is not yet
+        fixed): capture on the first real batch, or call reset_controller()
+        afterwards."""
         side = torch.cuda.Stream(device=self.lse.device)
         side.wait_stream(torch.cuda.current_stream(self.lse.device))
         with torch.cuda.stream(side):           # one eager run on the capture stream first
