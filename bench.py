@@ -26,7 +26,13 @@ import sys
 import threading
 import time
 
-import numpy as np
+# The CPU oracle legs are timed on one thread and report cores = 1: keep
+# numpy's BLAS (the LM-head projection's matrix product) to one thread too.
+# Set before numpy is imported, which is when the BLAS library reads them.
+for _v in ("OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")
+
+import numpy as np  # noqa: E402
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
