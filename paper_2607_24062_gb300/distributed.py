@@ -30,11 +30,13 @@ def allreduce_batch_stats(batch: torch.Tensor, group=None) -> None:
     bytes, on the device the backend uses) over the ranks, in place."""
     if not dist.is_initialized() or dist.get_world_size(group) == 1:
         return
-    for name, dtype in (("n_tokens", torch.int64), ("n_groups_valid", torch.int32), ("Y_sum", torch.float64)):
-        view = _field(batch, name, dtype)
-        tmp = view.clone()
-        dist.all_reduce(tmp, op=dist.ReduceOp.SUM, group=group)
-        view.copy_(tmp)
+    # one collective: the two counts travel as float64 (exact below 2^53) beside the sum
+    fields = (("n_tokens", torch.int64), ("n_groups_valid", torch.int32), ("Y_sum", torch.float64))
+    views = [_field(batch, name, dtype) for name, dtype in fields]
+    packed = torch.stack([v.reshape(()).to(torch.float64) for v in views])
+    dist.all_reduce(packed, op=dist.ReduceOp.SUM, group=group)
+    for k, v in enumerate(views):
+        v.copy_(packed[k].to(v.dtype))
 
 
 def shard_seed(base_seed: int, rank: int) -> int:
