@@ -130,6 +130,36 @@ def _round_bf16_truncates(x):
     return np.ldexp(np.trunc(f * 256.0) / 256.0, e)
 
 
+def _grpo_singleton_zero(rewards, group_offsets, params):
+    """Mistake: a prompt with one response gets A = 0 under the mean-0/std-1 rule."""
+    p = O.Params(**{**vars(params), "singleton_rule": O.SINGLETON_ZERO})
+    return OA._orig["grpo_advantage"](rewards, group_offsets, p)
+
+
+def _controller_zero_alpha_unguarded(state, params, lr, mask, so, go, seq, grp, batch, adv):
+    """Mistake: rho^alpha evaluated as exp(alpha * lr) with no alpha = 0 case, so that
+    alpha = 0 on a token with lr = +inf gives exp(0 * inf) = NaN instead of 1."""
+    w, alpha, st, info, f = OA._orig["controller_step"](state, params, lr, mask, so, go, seq, grp, batch, adv)
+    w = np.array(w, dtype=np.float64)
+    lr = np.asarray(lr, dtype=np.float64)
+    for i in range(len(so) - 1):
+        for t in range(int(so[i]), int(so[i + 1])):
+            valid = mask is None or mask[t] != 0
+            if valid and params.mode != O.MODE_MIS and alpha[i] == 0.0 and np.isinf(lr[t]):
+                w[t] = np.nan
+    return w, alpha, st, info, f
+
+
+def _controller_nan_weight_one(state, params, lr, mask, so, go, seq, grp, batch, adv):
+    """Mistake: a token whose log-ratio is NaN keeps weight 1 instead of 0."""
+    w, alpha, st, info, f = OA._orig["controller_step"](state, params, lr, mask, so, go, seq, grp, batch, adv)
+    w = np.array(w, dtype=np.float64)
+    lr = np.asarray(lr, dtype=np.float64)
+    nan = np.isnan(lr) if mask is None else np.isnan(lr) & (np.asarray(mask) != 0)
+    w[nan] = 1.0
+    return w, alpha, st, info, f
+
+
 PIN_GROUPS = {
     "token_stats": [lambda: P.test_token_stats_matches_bruteforce(7), P.test_token_stats_library_routines,
                     P.test_two_way_closed_form],
@@ -141,7 +171,7 @@ PIN_GROUPS = {
                         P.test_controller_special_cases, P.test_tis_and_mis_thresholds,
                         lambda: [P.test_continuous_reduction_always_reduces(r) for r in P._read_quadrants()],
                         P.test_continuous_reduction_kappa, P.test_moving_average_X_by_hand,
-                        P.test_calibration_averages_prompts_across_batches],
+                        P.test_calibration_averages_prompts_across_batches, P.test_infinite_and_nan_log_ratios],
     "loss_grad_logits": [lambda: P.test_gradient_matches_autograd(False, 0.0), P.test_on_policy_loss_by_hand_and_invariants,
                          lambda: P.test_gradient_central_differences(0.0), P.test_entropy_bonus_by_hand],
     "round_bf16": [P.test_round_bf16_matches_library_and_ties],
@@ -166,6 +196,9 @@ MUTATIONS = [
     ("loss_grad_logits", "entropy bonus with the wrong sign", _loss_grad_entropy_sign),
     ("seq_discrepancy", "Y_g weighted by tokens instead of responses", _discrepancy_token_weighted_Y),
     ("lmhead_logits", "logits not rounded to bf16", _lmhead_not_rounded),
+    ("grpo_advantage", "lone response given no advantage", _grpo_singleton_zero),
+    ("controller_step", "alpha = 0 with an infinite log-ratio gives NaN", _controller_zero_alpha_unguarded),
+    ("controller_step", "NaN log-ratio keeps weight 1", _controller_nan_weight_one),
 ]
 
 
