@@ -160,6 +160,13 @@ def _controller_nan_weight_one(state, params, lr, mask, so, go, seq, grp, batch,
     return w, alpha, st, info, f
 
 
+def _loss_grad_no_clip(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch, params, rows=None):
+    """Mistake: the PPO clip left out (min(r A, clip(r) A) taken as r A everywhere)."""
+    p = O.Params(**{**vars(params), "clip_eps": 1e9})
+    return OA._orig["loss_grad_logits"](z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch, p,
+                                        rows)
+
+
 PIN_GROUPS = {
     "token_stats": [lambda: P.test_token_stats_matches_bruteforce(7), P.test_token_stats_library_routines,
                     P.test_two_way_closed_form],
@@ -173,7 +180,8 @@ PIN_GROUPS = {
                         P.test_continuous_reduction_kappa, P.test_moving_average_X_by_hand,
                         P.test_calibration_averages_prompts_across_batches, P.test_infinite_and_nan_log_ratios],
     "loss_grad_logits": [lambda: P.test_gradient_matches_autograd(False, 0.0), P.test_on_policy_loss_by_hand_and_invariants,
-                         lambda: P.test_gradient_central_differences(0.0), P.test_entropy_bonus_by_hand],
+                         lambda: P.test_gradient_central_differences(0.0), P.test_entropy_bonus_by_hand,
+                         lambda: P.test_gradient_matches_autograd(True, 0.0), P.test_clip_gate],
     "round_bf16": [P.test_round_bf16_matches_library_and_ties],
     "lmhead_logits": [P.test_lmhead_logits_small],
 }
@@ -199,6 +207,7 @@ MUTATIONS = [
     ("grpo_advantage", "lone response given no advantage", _grpo_singleton_zero),
     ("controller_step", "alpha = 0 with an infinite log-ratio gives NaN", _controller_zero_alpha_unguarded),
     ("controller_step", "NaN log-ratio keeps weight 1", _controller_nan_weight_one),
+    ("loss_grad_logits", "PPO clip left out", _loss_grad_no_clip),
 ]
 
 
