@@ -167,6 +167,21 @@ def _loss_grad_no_clip(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, se
                                         rows)
 
 
+def _controller_y_per_response(state, params, *args):
+    """Mistake: Y read per response (D_i) where the prompt mean Y_g is the default."""
+    if params.y_gran == O.Y_GROUP:
+        params = O.Params(**{**vars(params), "y_gran": O.Y_SEQUENCE})
+    return OA._orig["controller_step"](state, params, *args)
+
+
+def _controller_mis_mean_ratio(state, params, lr, mask, so, go, seq, grp, batch, adv):
+    """Mistake: the sequence ratio of MIS from the mean token log-ratio instead of the sum."""
+    seq2 = dict(seq)
+    n = np.maximum(np.asarray(seq["n"]), 1)
+    seq2["sum_lr"] = np.asarray(seq["sum_lr"], dtype=np.float64) / n
+    return OA._orig["controller_step"](state, params, lr, mask, so, go, seq2, grp, batch, adv)
+
+
 PIN_GROUPS = {
     "token_stats": [lambda: P.test_token_stats_matches_bruteforce(7), P.test_token_stats_library_routines,
                     P.test_two_way_closed_form],
@@ -178,7 +193,8 @@ PIN_GROUPS = {
                         P.test_controller_special_cases, P.test_tis_and_mis_thresholds,
                         lambda: [P.test_continuous_reduction_always_reduces(r) for r in P._read_quadrants()],
                         P.test_continuous_reduction_kappa, P.test_moving_average_X_by_hand,
-                        P.test_calibration_averages_prompts_across_batches, P.test_infinite_and_nan_log_ratios],
+                        P.test_calibration_averages_prompts_across_batches, P.test_infinite_and_nan_log_ratios,
+                        P.test_y_granularity_options, P.test_mis_sequence_ratio_is_product],
     "loss_grad_logits": [lambda: P.test_gradient_matches_autograd(False, 0.0), P.test_on_policy_loss_by_hand_and_invariants,
                          lambda: P.test_gradient_central_differences(0.0), P.test_entropy_bonus_by_hand,
                          lambda: P.test_gradient_matches_autograd(True, 0.0), P.test_clip_gate],
@@ -208,6 +224,8 @@ MUTATIONS = [
     ("controller_step", "alpha = 0 with an infinite log-ratio gives NaN", _controller_zero_alpha_unguarded),
     ("controller_step", "NaN log-ratio keeps weight 1", _controller_nan_weight_one),
     ("loss_grad_logits", "PPO clip left out", _loss_grad_no_clip),
+    ("controller_step", "Y per response instead of per prompt", _controller_y_per_response),
+    ("controller_step", "MIS ratio from the mean log-ratio", _controller_mis_mean_ratio),
 ]
 
 

@@ -285,13 +285,14 @@ def test_tis_and_mis_thresholds():
 
 def test_mis_sequence_ratio_is_product():
     # rho_i = prod_t pi/mu over the valid tokens of the response (Eq. MIS)
+    # (a product away from 1, so that a mean of the log-ratios or a single token's ratio cannot pass)
     pi = np.array([0.5, 0.2, 0.9, 0.3])
-    mu = np.array([0.4, 0.25, 0.9, 0.1])
+    mu = np.array([0.4, 0.5, 0.6, 0.1])
     mask = np.array([1, 1, 1, 0])
     lr, d, seq, grp, batch, _ = O.seq_discrepancy(np.log(pi), np.log(mu), mask, [0, 4], [0, 1])
     p = O.Params(mode=O.MODE_MIS, X_init=1.0)
     w, *_ = O.controller_step(O.controller_init(p), p, lr, mask, [0, 4], [0, 1], seq, grp, batch, [1.0])
-    prod = (0.5 / 0.4) * (0.2 / 0.25) * (0.9 / 0.9)
+    prod = (0.5 / 0.4) * (0.2 / 0.5) * (0.9 / 0.6)   # 0.75, the masked token left out
     np.testing.assert_allclose(w, [prod, prod, prod, 0.0], rtol=1e-14)
 
 
