@@ -182,6 +182,68 @@ def _controller_mis_mean_ratio(state, params, lr, mask, so, go, seq, grp, batch,
     return OA._orig["controller_step"](state, params, lr, mask, so, go, seq2, grp, batch, adv)
 
 
+def _token_stats_lse_without_max(z, ids, mask):
+    """Mistake: the row maximum subtracted for stability never added back."""
+    lse, logp, H, f = OA._orig["token_stats"](z, ids, mask)
+    mx = np.asarray(z, dtype=np.float64).max(axis=1)
+    m = np.ones(len(lse), dtype=bool) if mask is None else np.asarray(mask) != 0
+    return np.where(m, lse - mx, lse), np.where(m, logp + mx, logp), np.where(m, H - mx, H), f
+
+
+def _regroup(seq, grp, go, divisor):
+    for g in range(len(go) - 1):
+        members = list(range(go[g], go[g + 1]))
+        valid = [i for i in members if seq["n"][i] > 0]
+        den = divisor(members, valid)
+        grp["Y"][g] = sum(seq["mean_d"][i] for i in valid) / den if den else 0.0
+
+
+def _discrepancy_mean_over_all_rows(logp_pi, logp_mu, mask, so, go, entropy=None):
+    """Mistake: D_i divides by every row of the response, masked padding included."""
+    lr, d, seq, grp, batch, f = OA._orig["seq_discrepancy"](logp_pi, logp_mu, mask, so, go, entropy)
+    so = np.asarray(so)
+    for i in range(len(so) - 1):
+        if seq["n"][i] > 0:
+            seq["mean_d"][i] = seq["sum_d"][i] / (so[i + 1] - so[i])
+    _regroup(seq, grp, go, lambda members, valid: len(valid))
+    return lr, d, seq, grp, batch, f
+
+
+def _discrepancy_empty_responses_counted(logp_pi, logp_mu, mask, so, go, entropy=None):
+    """Mistake: G_g counts the responses with no valid token."""
+    lr, d, seq, grp, batch, f = OA._orig["seq_discrepancy"](logp_pi, logp_mu, mask, so, go, entropy)
+    _regroup(seq, grp, go, lambda members, valid: len(members) if valid else 0)
+    return lr, d, seq, grp, batch, f
+
+
+def _grpo_no_eps(rewards, group_offsets, params):
+    """Mistake: adv_eps left out of the denominator."""
+    return OA._orig["grpo_advantage"](rewards, group_offsets, O.Params(**{**vars(params), "adv_eps": 0.0}))
+
+
+def _controller_never_frozen(state, params, *args):
+    """Mistake: X recalibrated on every batch instead of frozen after calibration."""
+    if params.X_init <= 0 and state.calibrated:
+        state.calibrated = False
+        state.calib_sum, state.calib_count, state.calib_done_steps = 0.0, 0, 0
+    return OA._orig["controller_step"](state, params, *args)
+
+
+def _loss_grad_token_mean(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch, params, rows=None):
+    """Mistake: the default sequence-mean-token-mean aggregation replaced by a token mean."""
+    if params.agg == O.AGG_SEQ_MEAN_TOKEN_MEAN:
+        params = O.Params(**{**vars(params), "agg": O.AGG_TOKEN_MEAN})
+    return OA._orig["loss_grad_logits"](z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch,
+                                        params, rows)
+
+
+def _round_bf16_half_away(x):
+    """Mistake: ties rounded away from zero instead of to even."""
+    x = np.asarray(x, dtype=np.float64)
+    f, e = np.frexp(x)
+    return np.ldexp(np.trunc(f * 256.0 + np.copysign(0.5, f)) / 256.0, e)
+
+
 PIN_GROUPS = {
     "token_stats": [lambda: P.test_token_stats_matches_bruteforce(7), P.test_token_stats_library_routines,
                     P.test_two_way_closed_form],
@@ -194,7 +256,8 @@ PIN_GROUPS = {
                         lambda: [P.test_continuous_reduction_always_reduces(r) for r in P._read_quadrants()],
                         P.test_continuous_reduction_kappa, P.test_moving_average_X_by_hand,
                         P.test_calibration_averages_prompts_across_batches, P.test_infinite_and_nan_log_ratios,
-                        P.test_y_granularity_options, P.test_mis_sequence_ratio_is_product],
+                        P.test_y_granularity_options, P.test_mis_sequence_ratio_is_product,
+                        P.test_calibration_then_frozen],
     "loss_grad_logits": [lambda: P.test_gradient_matches_autograd(False, 0.0), P.test_on_policy_loss_by_hand_and_invariants,
                          lambda: P.test_gradient_central_differences(0.0), P.test_entropy_bonus_by_hand,
                          lambda: P.test_gradient_matches_autograd(True, 0.0), P.test_clip_gate],
@@ -226,6 +289,13 @@ MUTATIONS = [
     ("loss_grad_logits", "PPO clip left out", _loss_grad_no_clip),
     ("controller_step", "Y per response instead of per prompt", _controller_y_per_response),
     ("controller_step", "MIS ratio from the mean log-ratio", _controller_mis_mean_ratio),
+    ("token_stats", "row maximum never added back to lse", _token_stats_lse_without_max),
+    ("seq_discrepancy", "D_i over every row, padding included", _discrepancy_mean_over_all_rows),
+    ("seq_discrepancy", "empty responses counted in G_g", _discrepancy_empty_responses_counted),
+    ("grpo_advantage", "adv_eps left out", _grpo_no_eps),
+    ("controller_step", "X recalibrated every batch", _controller_never_frozen),
+    ("loss_grad_logits", "token mean instead of sequence mean", _loss_grad_token_mean),
+    ("round_bf16", "ties away from zero", _round_bf16_half_away),
 ]
 
 

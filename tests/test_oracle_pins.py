@@ -189,6 +189,10 @@ def test_grpo_binary_closed_form(G, k):
     std = math.sqrt(k * (G - k) / (G * (G - 1)))
     np.testing.assert_allclose(A[:k], (1 - k / G) / std, rtol=1e-13)
     np.testing.assert_allclose(A[k:], -(k / G) / std, rtol=1e-13)
+    # the epsilon is added to the standard deviation (reading of the A formula under Eq. grpo_objective)
+    A = O.grpo_advantage(R, [0, G], O.Params(adv_eps=0.25))
+    np.testing.assert_allclose(A[:k], (1 - k / G) / (std + 0.25), rtol=1e-13)
+    np.testing.assert_allclose(A[k:], -(k / G) / (std + 0.25), rtol=1e-13)
 
 
 def test_grpo_matches_scipy_zscore():
@@ -459,7 +463,7 @@ def test_gradient_matches_autograd(with_old, beta):
     L = _torch_loss(zt, f, p)
     L.backward()
     np.testing.assert_allclose(grad, zt.grad.numpy(), atol=1e-14)
-    assert loss == pytest.approx(float(L), abs=1e-14)
+    assert loss == pytest.approx(float(L.detach()), abs=1e-14)
 
 
 @pytest.mark.parametrize("beta", [0.0, 0.3])
