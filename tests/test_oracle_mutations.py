@@ -244,11 +244,29 @@ def _round_bf16_half_away(x):
     return np.ldexp(np.trunc(f * 256.0 + np.copysign(0.5, f)) / 256.0, e)
 
 
+def _token_stats_no_bad_id_flag(z, ids, mask):
+    """Mistake: an id outside [0, V) is not reported."""
+    lse, logp, H, f = OA._orig["token_stats"](z, ids, mask)
+    return lse, logp, H, f & ~O.FLAG_BAD_ID
+
+
+def _discrepancy_no_offsets_flag(logp_pi, logp_mu, mask, so, go, entropy=None):
+    """Mistake: inconsistent offsets are not reported."""
+    lr, d, seq, grp, batch, f = OA._orig["seq_discrepancy"](logp_pi, logp_mu, mask, so, go, entropy)
+    return lr, d, seq, grp, batch, f & ~O.FLAG_BAD_OFFSETS
+
+
+def _controller_no_x_flag(state, params, *args):
+    """Mistake: X <= 0 is not reported."""
+    w, alpha, st, info, f = OA._orig["controller_step"](state, params, *args)
+    return w, alpha, st, info, f & ~O.FLAG_X_NONPOS
+
+
 PIN_GROUPS = {
     "token_stats": [lambda: P.test_token_stats_matches_bruteforce(7), P.test_token_stats_library_routines,
-                    P.test_two_way_closed_form],
+                    P.test_two_way_closed_form, P.test_mask_nonfinite_and_bad_id],
     "seq_discrepancy": [P.test_distance_is_on_probabilities, P.test_hand_worked_aggregates,
-                        P.test_aggregates_as_linear_functional],
+                        P.test_aggregates_as_linear_functional, P.test_bad_offsets_flagged],
     "grpo_advantage": [lambda: P.test_grpo_binary_closed_form(8, 3), P.test_grpo_matches_scipy_zscore,
                        P.test_grpo_special_groups],
     "controller_step": [lambda: [P.test_quadrant_sign_table(r) for r in P._read_quadrants()],
@@ -257,7 +275,7 @@ PIN_GROUPS = {
                         P.test_continuous_reduction_kappa, P.test_moving_average_X_by_hand,
                         P.test_calibration_averages_prompts_across_batches, P.test_infinite_and_nan_log_ratios,
                         P.test_y_granularity_options, P.test_mis_sequence_ratio_is_product,
-                        P.test_calibration_then_frozen],
+                        P.test_calibration_then_frozen, P.test_nonpositive_X_flag_and_fixed_point],
     "loss_grad_logits": [lambda: P.test_gradient_matches_autograd(False, 0.0), P.test_on_policy_loss_by_hand_and_invariants,
                          lambda: P.test_gradient_central_differences(0.0), P.test_entropy_bonus_by_hand,
                          lambda: P.test_gradient_matches_autograd(True, 0.0), P.test_clip_gate],
@@ -296,6 +314,9 @@ MUTATIONS = [
     ("controller_step", "X recalibrated every batch", _controller_never_frozen),
     ("loss_grad_logits", "token mean instead of sequence mean", _loss_grad_token_mean),
     ("round_bf16", "ties away from zero", _round_bf16_half_away),
+    ("token_stats", "bad id not reported", _token_stats_no_bad_id_flag),
+    ("seq_discrepancy", "bad offsets not reported", _discrepancy_no_offsets_flag),
+    ("controller_step", "X <= 0 not reported", _controller_no_x_flag),
 ]
 
 
