@@ -30,7 +30,8 @@
  *     row stride `ld` in elements; the base pointer must be 16-byte aligned
  *     and ld a multiple of 8, so every row starts on a 16-byte boundary.
  *   - Sizes: 1 <= V <= 2^30 (column indices stay in 32-bit range); the row
- *     count T is 64-bit (T * ld may exceed 2^32).  Larger V is
+ *     count T is 64-bit (T and T * ld may exceed 2^32); a response holds
+ *     fewer than 2^31 tokens (its count is an int32).  Larger V is
  *     ACRL_ERR_INVALID_ARG.
  *
  * Notation: T token rows, V vocabulary size, S responses (sequences),
