@@ -367,9 +367,9 @@ acrl_status acrl_lmhead_logits_stats(const acrl_bf16* hidden, int64_t M, int64_t
 
 /*
  * acrl_lmhead_merge -- lse, logp = z[a] - lse and entropy per row from the
- * partial states of acrl_lmhead_logits_stats (tiles merged in order, so the
- * result is deterministic); same outputs, masking and flags as
- * acrl_token_stats.  z[a] is read from `logits`.
+ * partial states of acrl_lmhead_logits_stats (the tiles of a row combined in
+ * a fixed order, so the result is deterministic); same outputs, masking and
+ * flags as acrl_token_stats.  z[a] is read from `logits`.
  */
 acrl_status acrl_lmhead_merge(const float* partials, const acrl_bf16* logits, int64_t M, int64_t N,
                               int64_t ldl, const int32_t* ids, const uint8_t* mask,
