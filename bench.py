@@ -495,10 +495,8 @@ def _weight_calls_ms(acrl, W, dev, median_ms):
     flags = acrl.api.new_flags(dev)
 
     def calls():
-        disc = acrl.seq_discrepancy(d["logp_pi"], d["logp_mu"], d["mask"], d["seq_offsets"], d["group_offsets"],
-                                    flags=flags)
-        adv = acrl.grpo_advantage(d["rewards"], d["group_offsets"], p, flags=flags)
-        acrl.controller_step(state, p, disc, d["mask"], d["seq_offsets"], d["group_offsets"], adv, flags=flags)
+        acrl.importance_weights(state, p, d["logp_pi"], d["logp_mu"], d["mask"], d["rewards"], d["seq_offsets"],
+                                d["group_offsets"], flags=flags)
 
     ms = median_ms(calls, 20)
     return {"ms": ms, "tokens": int(d["mask"].sum()), "rows": d["T"], "flags": acrl.read_flags(flags),

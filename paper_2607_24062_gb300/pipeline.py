@@ -14,6 +14,7 @@ to a callback.
 
 from __future__ import annotations
 
+from dataclasses import dataclass
 from typing import Callable
 
 import torch
@@ -137,3 +138,32 @@ class AcrlStep:
 
     def state_host(self):
         return api.read_state(self.state)
+
+
+@dataclass
+class Weights:
+    weight: torch.Tensor      # float32 [T] importance weight per token (0 where masked)
+    coef: torch.Tensor        # float32 [T] loss coefficient m w A / norm per token
+    adv: torch.Tensor         # float32 [S] GRPO advantage per response
+    alpha: torch.Tensor       # float32 [S] controller exponent per response
+    disc: api.Discrepancy     # lr, d and the per-response / per-prompt / batch statistics
+    flags: torch.Tensor       # int32 [1] device flags word of the three calls
+
+
+def importance_weights(state, params: Params, logp_old, logp_mu, mask, rewards, seq_offsets, group_offsets, *,
+                       exchange: Callable[[torch.Tensor], None] | None = None, flags=None, stream=None) -> Weights:
+    """The weights of one batch from per-token log-probs alone: the old
+    policy's log-probs of the sampled tokens and the rollout engine's (the
+    call whose cost Sec. 5.4 reports), i.e. seq_discrepancy, grpo_advantage
+    and controller_step in order on one stream.  `state` is the controller
+    state (api.controller_init), advanced in place; `exchange` is applied to
+    the batch-statistics bytes before the controller, as in
+    AcrlStep.statistics."""
+    flags = api.new_flags(logp_old.device) if flags is None else flags
+    disc = api.seq_discrepancy(logp_old, logp_mu, mask, seq_offsets, group_offsets, flags=flags, stream=stream)
+    if exchange is not None:
+        exchange(disc.batch)
+    adv = api.grpo_advantage(rewards, group_offsets, params, flags=flags, stream=stream)
+    weight, coef, alpha = api.controller_step(state, params, disc, mask, seq_offsets, group_offsets, adv, flags=flags,
+                                              stream=stream)
+    return Weights(weight, coef, adv, alpha, disc, flags)

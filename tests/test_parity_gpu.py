@@ -648,3 +648,32 @@ def test_infinite_and_nan_rollout_log_probs_on_gpu():
         assert api.read_flags(flags) & acrl.FLAG_NONFINITE and of & O.FLAG_NONFINITE
         np.testing.assert_allclose(host(w), ow, rtol=1e-6, atol=0, err_msg=f"mode {mode}")
         assert host(w)[2] == 0.0
+
+
+@pytest.mark.parametrize("mode", [acrl.MODE_ACRL, acrl.MODE_MIS])
+def test_importance_weights_from_log_probs(mode):
+    """The weights-only call (log-probs in, weights out) against the oracle's
+    discrepancy, advantage and controller stages, over three batches (the
+    first calibrates X)."""
+    spec = W.small_variant(W.GRPO, name="weights_only", n_prompts=4, group_size=4, len_lo=5, len_hi=90,
+                           perturb_frac=0.3, perturb_std=0.3)
+    p = acrl.Params(mode=mode)
+    op = oracle_params(p)
+    state, ostate = api.controller_init(p), O.controller_init(op)
+    for k in range(3):
+        d = W.token_level(spec, 700 + k, device=DEV)
+        r = acrl.importance_weights(state, p, d["logp_pi"], d["logp_mu"], d["mask"], d["rewards"], d["seq_offsets"],
+                                    d["group_offsets"])
+        mask, so, go = host(d["mask"]), host(d["seq_offsets"]), host(d["group_offsets"])
+        lr, dd, seq, grp, batch, f = O.seq_discrepancy(host(d["logp_pi"]).astype(np.float64),
+                                                        host(d["logp_mu"]).astype(np.float64), mask, so, go)
+        adv = O.grpo_advantage(host(d["rewards"]).astype(np.float64), go, op)
+        w, alpha, ostate, info, f2 = O.controller_step(ostate, op, lr, mask, so, go, seq, grp, batch, adv)
+        assert api.read_flags(r.flags) == (f | f2)
+        compare_seq(r.disc.seq_host(), seq)
+        assert_close_rel(host(r.adv), adv, floor=1e-6, what="adv")
+        assert_close_rel(host(r.alpha), alpha, floor=1e-6, what="alpha")
+        assert_close_rel(host(r.weight), w, floor=1e-7, what="weight")
+        coef = O.loss_coefficients(w, adv, mask, so, seq, grp, batch, op)
+        assert_close_rel(host(r.coef), coef, floor=1e-12, what="coef")
+        assert_close_rel(api.read_state(state)["X"], ostate.X, floor=1e-12, what="X")
