@@ -41,3 +41,13 @@ def test_c_client_device_call(tmp_path):
                    libs=(f"-L{cuda}/lib64", "-lcudart", f"-Wl,-rpath,{cuda}/lib64"))
     r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
     assert r.returncode == 0 and r.stdout.strip() == "ok", r.stdout + r.stderr
+
+
+@pytest.mark.gpu
+def test_c_client_whole_chain(tmp_path):
+    """The whole on-policy pass through the C ABI alone, checked in C."""
+    cuda = os.environ.get("CUDA_HOME", "/usr/local/cuda")
+    exe = _compile(tmp_path, "abi_chain.c", cflags=("-isystem", f"{cuda}/include"),
+                   libs=(f"-L{cuda}/lib64", "-lcudart", f"-Wl,-rpath,{cuda}/lib64"))
+    r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
+    assert r.returncode == 0 and r.stdout.strip() == "ok", r.stdout + r.stderr
