@@ -254,6 +254,20 @@ acrl_status acrl_grpo_advantage(const float* rewards, const int32_t* group_offse
 acrl_status acrl_controller_init(acrl_controller_state* state, const acrl_params* p, acrl_stream stream);
 
 /*
+ * acrl_controller_save / acrl_controller_load -- copy the controller state
+ * between its device location and host memory: a checkpoint of the only
+ * state the method carries from step to step (X and its calibration, fixed
+ * once calibrated, Sec. 4.1).  Resuming from a saved state is bit-exact.
+ *   state       device acrl_controller_state.
+ *   host_state  host memory of one acrl_controller_state (any alignment).
+ * Both are ordered on `stream` and synchronise it before returning.
+ */
+acrl_status acrl_controller_save(const acrl_controller_state* state, acrl_controller_state* host_state,
+                                 acrl_stream stream);
+acrl_status acrl_controller_load(acrl_controller_state* state, const acrl_controller_state* host_state,
+                                 acrl_stream stream);
+
+/*
  * acrl_controller_step -- the adaptive controller and the importance weights.
  * Calibration (Sec. 4.1, X fixed before training; Sec. 5.1 takes it from
  * step 0): while not calibrated, Y_sum and Q_eff of `batch` are added to the

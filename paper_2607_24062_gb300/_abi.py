@@ -66,6 +66,8 @@ SIGNATURES = {
                                      c_p, c_p]),
     "acrl_grpo_advantage": (c_i32, [c_p, c_p, c_i32, c_i32, ctypes.POINTER(Params), c_p, c_p, c_p]),
     "acrl_controller_init": (c_i32, [c_p, ctypes.POINTER(Params), c_p]),
+    "acrl_controller_save": (c_i32, [c_p, c_p, c_p]),
+    "acrl_controller_load": (c_i32, [c_p, c_p, c_p]),
     "acrl_controller_step": (c_i32, [c_p, ctypes.POINTER(Params), c_p, c_p, c_i64, c_p, c_i32, c_p, c_i32, c_p, c_p,
                                      c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p]),
     "acrl_loss_grad_logits": (c_i32, [c_p, c_i64, c_i64, c_i64, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_f32, c_p, c_p,

@@ -182,19 +182,24 @@ def read_state(state: torch.Tensor) -> np.void:
     return read_structs(state, STATE_DTYPE, 1)[0]
 
 
-def save_state(state: torch.Tensor) -> bytes:
-    """The controller state's 48 bytes, for a checkpoint (the state is plain data)."""
-    return bytes(state[: STATE_DTYPE.itemsize].cpu().numpy().tobytes())
+def save_state(state: torch.Tensor, stream=None) -> bytes:
+    """acrl_controller_save: the controller state's 48 bytes, for a checkpoint
+    (the state is plain data)."""
+    _need(state, torch.uint8, STATE_DTYPE.itemsize, "state")
+    buf = ctypes.create_string_buffer(STATE_DTYPE.itemsize)
+    _call("acrl_controller_save", (state,), stream, _ptr(state), ctypes.addressof(buf))
+    return buf.raw
 
 
-def load_state(blob: bytes, state: torch.Tensor | None = None, device=None) -> torch.Tensor:
-    """Restore a controller state saved by save_state; resuming from it is bit-exact."""
+def load_state(blob: bytes, state: torch.Tensor | None = None, device=None, stream=None) -> torch.Tensor:
+    """acrl_controller_load: restore a state saved by save_state; resuming
+    from it is bit-exact."""
     if len(blob) != STATE_DTYPE.itemsize:
         raise AcrlError("controller state: wrong size")
-    host = torch.frombuffer(bytearray(blob), dtype=torch.uint8)
-    if state is None:
-        state = struct_buffer(STATE_DTYPE, 1, device)
-    state[: STATE_DTYPE.itemsize].copy_(host)
+    state = struct_buffer(STATE_DTYPE, 1, device) if state is None else \
+        _need(state, torch.uint8, STATE_DTYPE.itemsize, "state")
+    buf = ctypes.create_string_buffer(bytes(blob), STATE_DTYPE.itemsize)
+    _call("acrl_controller_load", (state,), stream, _ptr(state), ctypes.addressof(buf))
     return state
 
 

@@ -424,6 +424,24 @@ extern "C" acrl_status acrl_controller_init(acrl_controller_state* state, const 
     return launch_status();
 }
 
+extern "C" acrl_status acrl_controller_save(const acrl_controller_state* state, acrl_controller_state* host_state,
+                                            acrl_stream stream) {
+    if (!state || !host_state) return ACRL_ERR_INVALID_ARG;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(host_state, state, sizeof(acrl_controller_state), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return ACRL_ERR_CUDA;
+    return cudaStreamSynchronize(s) == cudaSuccess ? ACRL_OK : ACRL_ERR_CUDA;
+}
+
+extern "C" acrl_status acrl_controller_load(acrl_controller_state* state, const acrl_controller_state* host_state,
+                                            acrl_stream stream) {
+    if (!state || !host_state) return ACRL_ERR_INVALID_ARG;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(state, host_state, sizeof(acrl_controller_state), cudaMemcpyHostToDevice, s) != cudaSuccess)
+        return ACRL_ERR_CUDA;
+    return cudaStreamSynchronize(s) == cudaSuccess ? ACRL_OK : ACRL_ERR_CUDA;
+}
+
 extern "C" acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params* p, const float* lr,
                                             const uint8_t* mask, int64_t T, const int64_t* seq_offsets, int32_t S,
                                             const int32_t* group_offsets, int32_t Gn, acrl_seq_stats* seq,

@@ -6,7 +6,8 @@
  * ACRL weight is 1; the advantages of rewards (1, 0) are +-0.5 / (sqrt(0.5) +
  * adv_eps), the loss coefficients A_i / (Q G n_i), and the gradient
  * coef (p - onehot), all checked against double-precision values computed
- * here.  Prints "ok". */
+ * here; the controller state is saved to the host and restored.  Prints
+ * "ok". */
 #include <math.h>
 #include <stdio.h>
 #include <string.h>
@@ -114,6 +115,19 @@ int main(void) {
     CHECK(acrl_loss_grad_logits(d_logits, T, V, LD, d_ids, d_mask, d_lse, NULL, d_coef, NULL, NULL, p.clip_eps, d_grad,
                                 d_tl, d_loss, d_flags, NULL));
     CHECK(acrl_check_flags(d_flags, NULL));
+    {   /* checkpoint the controller and restore it into a fresh device state */
+        acrl_controller_state saved, again;
+        void* d_state2 = NULL;
+        CHECK(acrl_controller_save(d_state, &saved, NULL));
+        if (cudaMalloc(&d_state2, sizeof saved) != cudaSuccess) return 2;
+        CHECK(acrl_controller_load(d_state2, &saved, NULL));
+        CHECK(acrl_controller_save(d_state2, &again, NULL));
+        cudaFree(d_state2);
+        if (saved.X != 0.013 || saved.calibrated != 1 || saved.step != 1 || memcmp(&saved, &again, sizeof saved)) {
+            fprintf(stderr, "controller checkpoint off\n");
+            return 1;
+        }
+    }
 
     cudaMemcpy(h_lse, d_lse, sizeof h_lse, cudaMemcpyDeviceToHost);
     cudaMemcpy(h_coef, d_coef, sizeof h_coef, cudaMemcpyDeviceToHost);

@@ -73,6 +73,8 @@ def test_host_side_rejections(L):
     assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(x_ema=1.5)), None) == E
     assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(entropy_coeff=-1.0)), None) == E
     assert L.acrl_read_flags(None, None, None) == E
+    assert L.acrl_controller_save(None, fake, None) == E and L.acrl_controller_save(fake, None, None) == E
+    assert L.acrl_controller_load(None, fake, None) == E and L.acrl_controller_load(fake, None, None) == E
     assert L.acrl_reduce_loss(None, 4, fake, None) == E
     assert L.acrl_selftest_wait_timeout(None, 1000, None) == E
     assert L.acrl_selftest_wait_timeout(fake, 3_000_000_000, None) == E
