@@ -137,3 +137,35 @@ def test_lmhead_workload_full_chain():
     ograd, _, _ = O.loss_grad_logits(zg, host(b.ids), mask, lse_full, None, oadv, ow, so, seq, grp, batch, op,
                                      rows=rows)
     assert_grad_rows(grad_rows(grad, rows, b.N), ograd, ocoef[rows], host(b.ids)[rows])
+
+
+def test_lmhead_flags_nonfinite_and_bad_id_rows_like_token_stats():
+    """A NaN in one hidden row makes that row's logits NaN: the merge gives NaN
+    lse/logp/entropy there and raises NONFINITE; an id outside [0, N) gives
+    logp = 0 and BAD_ID; every other row is unaffected.  Same outputs and flags
+    as acrl_token_stats on the stored logits."""
+    M, N, K = 130, 520, 64
+    gen = torch.Generator(device=DEV).manual_seed(11)
+    H = torch.randn((M, K), generator=gen, device=DEV).to(torch.bfloat16)
+    H[5, 17] = float("nan")
+    Wt = (0.02 * torch.randn((N, K), generator=gen, device=DEV)).to(torch.bfloat16)
+    ids = torch.randint(0, N, (M,), generator=gen, device=DEV, dtype=torch.int32)
+    ids[7] = N
+    flags = api.new_flags()
+    logits, partials = api.lmhead_logits_stats(H, Wt, N=N, flags=flags)
+    lse, logp, ent = api.lmhead_merge(partials, logits, ids, None, N=N, flags=flags)
+    f = api.read_flags(flags)
+    assert f == (acrl.FLAG_NONFINITE | acrl.FLAG_BAD_ID)
+    assert torch.isnan(logits[5, :N].float()).all() and not torch.isnan(logits[:5, :N].float()).any()
+    for t in (lse, logp, ent):
+        assert torch.isnan(t[5]) and torch.isfinite(t[:5]).all() and torch.isfinite(t[6:]).all()
+    assert float(logp[7]) == 0.0
+    flags2 = api.new_flags()
+    lse2, logp2, ent2 = api.token_stats(logits, ids, None, V=N, flags=flags2)
+    assert api.read_flags(flags2) == f
+    ok = torch.ones(M, dtype=torch.bool, device=DEV)
+    ok[5] = False
+    assert_close_abs(host(lse[ok]), host(lse2[ok]), 1e-5 + 1e-6 * np.abs(host(lse2[ok])), "lse")
+    assert_close_abs(host(logp[ok]), host(logp2[ok]), 2e-5, "logp")
+    assert_close_rel(host(ent[ok]), host(ent2[ok]), rel=1e-4, floor=1e-6, what="entropy")
+    assert torch.isnan(lse2[5]) and float(logp2[7]) == 0.0
