@@ -75,26 +75,47 @@ __device__ __forceinline__ uint4 grad_vec(const uint4 v, const RowPlan& rp, int 
 }
 
 // LAST: this is the second sweep over a row whose lines the first sweep kept in
-// L2, and the last read of them (L2 evict-first policy).
+// L2, and the last read of them (L2 evict-first policy).  It runs backwards,
+// so that it starts on the lines the first sweep loaded last, the ones most
+// likely still in L2.
 template <int TEAM, int UNROLL, bool ENT, bool LAST = false>
 __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ row, acrl_bf16* __restrict__ grow, int V,
                                                 int tid, const RowPlan& rp) {
     const int nvec = V >> 3;
     const uint4* src = reinterpret_cast<const uint4*>(row);
     uint4* dst = reinterpret_cast<uint4*>(grow);
-    const uint64_t pol = LAST ? policy_evict_first() : 0;
-    int v = tid;
-    for (; v + (UNROLL - 1) * TEAM < nvec; v += UNROLL * TEAM) {
-        uint4 buf[UNROLL];
+    if (LAST) {
+        const uint64_t pol = policy_evict_first();
+        // this thread's vectors are tid + i TEAM for i < mine; visit i = mine-1 down to 0
+        int i = tid < nvec ? (nvec - 1 - tid) / TEAM + 1 : 0;
+        for (; i >= UNROLL; i -= UNROLL) {
+            uint4 buf[UNROLL];
 #pragma unroll
-        for (int k = 0; k < UNROLL; ++k) buf[k] = LAST ? ld_policy(src + v + k * TEAM, pol) : ld_stream(src + v + k * TEAM);
+            for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(src + tid + (i - 1 - k) * TEAM, pol);
 #pragma unroll
-        for (int k = 0; k < UNROLL; ++k) {
-            const int vi = v + k * TEAM;
-            st_stream(dst + vi, grad_vec<ENT>(buf[k], rp, rp.a - (vi << 3)));
+            for (int k = 0; k < UNROLL; ++k) {
+                const int vi = tid + (i - 1 - k) * TEAM;
+                st_stream(dst + vi, grad_vec<ENT>(buf[k], rp, rp.a - (vi << 3)));
+            }
         }
+        for (; i > 0; --i) {
+            const int vi = tid + (i - 1) * TEAM;
+            st_stream(dst + vi, grad_vec<ENT>(ld_policy(src + vi, pol), rp, rp.a - (vi << 3)));
+        }
+    } else {
+        int v = tid;
+        for (; v + (UNROLL - 1) * TEAM < nvec; v += UNROLL * TEAM) {
+            uint4 buf[UNROLL];
+#pragma unroll
+            for (int k = 0; k < UNROLL; ++k) buf[k] = ld_stream(src + v + k * TEAM);
+#pragma unroll
+            for (int k = 0; k < UNROLL; ++k) {
+                const int vi = v + k * TEAM;
+                st_stream(dst + vi, grad_vec<ENT>(buf[k], rp, rp.a - (vi << 3)));
+            }
+        }
+        for (; v < nvec; v += TEAM) st_stream(dst + v, grad_vec<ENT>(ld_stream(src + v), rp, rp.a - (v << 3)));
     }
-    for (; v < nvec; v += TEAM) st_stream(dst + v, grad_vec<ENT>(ld_stream(src + v), rp, rp.a - (v << 3)));
     for (int j = (nvec << 3) + tid; j < V; j += TEAM) {
         float val = grad_elem<ENT>(bf16_to_float(row[j]), rp);
         if (!ENT && rp.sgn) val = -val;
