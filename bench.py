@@ -51,7 +51,7 @@ LAUNCHES_PER_STEP = 9
 # Taken with `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` (one pass) on the
 # bench workload; see profiles/dram_traffic_qwen_bench.md.
 NCU_TRAFFIC = {
-    "loss_grad.cu": {"src": "df650836df36a15e", "bytes_per_launch": 41.71e9 + 44.87e9},
+    "loss_grad.cu": {"src": "1726991a11c74fb9", "bytes_per_launch": 41.71e9 + 44.87e9},
     "token_stats.cu": {"src": "9e3bb1dc80555a69", "bytes_per_launch": 44.94e9 + 3.77e6},
 }
 
