@@ -51,8 +51,10 @@ LAUNCHES_PER_STEP = 9
 # Taken with `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` (one pass) on the
 # bench workload; see profiles/dram_traffic_qwen_bench.md.
 NCU_TRAFFIC = {
-    "loss_grad.cu": {"src": "1726991a11c74fb9", "bytes_per_launch": 41.71e9 + 44.87e9},
-    "token_stats.cu": {"src": "9e3bb1dc80555a69", "bytes_per_launch": 44.94e9 + 3.77e6},
+    "loss_grad.cu": {"src": "fabc7049c1e852c1", "bytes_per_launch": 41.71e9 + 44.87e9},
+    "token_stats.cu": {"src": "fa52d63034870905", "bytes_per_launch": 44.94e9 + 3.77e6},
+    # the LM-head GEMM at 32,768 x 4,096 x 151,936 (profiles/lmhead_kernel_lmhead_profile.md)
+    "lmhead.cu": {"src": "26ed7d7f20c2f3dd", "bytes_per_launch": 20.35e9 + 10.28e9},
 }
 
 
@@ -67,12 +69,20 @@ def _peaks():
 
 
 def _src_hash(name):
-    """Hash of a kernel source and the device headers it includes."""
+    """Hash of a kernel source and every header beside it."""
+    csrc = os.path.join(ROOT, "paper_2607_24062_gb300", "csrc")
+    headers = sorted(f for f in os.listdir(csrc) if f.endswith((".cuh", ".h")))
     d = hashlib.sha256()
-    for f in (name, "acrl_device.cuh", "row_lse.cuh", "acrl_host.h"):
-        with open(os.path.join(ROOT, "paper_2607_24062_gb300", "csrc", f), "rb") as fh:
+    for f in (name, *headers):
+        with open(os.path.join(csrc, f), "rb") as fh:
             d.update(fh.read())
     return d.hexdigest()[:16]
+
+
+def _traffic_of(name):
+    """ncu DRAM bytes per launch of a kernel source, if taken on the source as it is now."""
+    tr = NCU_TRAFFIC.get(name)
+    return tr["bytes_per_launch"] if tr and tr["src"] == _src_hash(name) else None
 
 
 class ClockSampler:
@@ -410,10 +420,7 @@ def run_ours(args):
     k1_avg = float(np.mean(k1_ms))
     k5_gbs = k5_bytes / (k5_avg / 1e3) / 1e9
     k1_gbs = k1_bytes / (k1_avg / 1e3) / 1e9
-    def traffic_of(name):
-        tr = NCU_TRAFFIC.get(name)
-        return tr["bytes_per_launch"] if tr and tr["src"] == _src_hash(name) else None
-    traffic = traffic_of("loss_grad.cu")
+    traffic = _traffic_of("loss_grad.cu")
 
     # the same step replayed from a CUDA graph (launch gaps removed); reported beside the eager step
     # (single process only: the multi-rank step keeps its collective outside any graph)
@@ -456,7 +463,7 @@ def run_ours(args):
                      "algorithmic_bytes_per_launch": k5_bytes, "ms_per_launch": k5_avg},
         "kernels": {
             "acrl_token_stats": {"ms": k1_avg, "GB/s": k1_gbs, "frac": k1_gbs / peak, "bytes": k1_bytes,
-                                 "traffic": traffic_of("token_stats.cu")},
+                                 "traffic": _traffic_of("token_stats.cu")},
             "acrl_loss_grad_logits": {"ms": k5_avg, "GB/s": k5_gbs, "frac": k5_gbs / peak, "bytes": k5_bytes},
             "seq_discrepancy+grpo_advantage+controller_step": {"ms": float(np.mean(mid_ms))},
             "acrl_loss_grad_logits (lse recomputed, cached-old)": {
@@ -587,8 +594,9 @@ def run_lmhead(args):
            "vs_baseline": None, "dtype": "bf16 (tensor cores, fp32 accumulate)", "data": "synthetic",
            "config": {"workload": _lmhead_desc(b), "flags": fl},
            "roofline": {"bound": "tensor", "kernel": "acrl_lmhead_logits_stats", "achieved": tf, "peak": peak,
-                        "unit": "TFLOP/s", "frac": tf / peak, "traffic": None, "peak_kind": kind,
-                        "flop_per_launch": flop, "ms_per_launch": gemm_ms},
+                        "unit": "TFLOP/s", "frac": tf / peak,
+                        "traffic": _traffic_of("lmhead.cu") if args.workload == "lmhead" else None,
+                        "peak_kind": kind, "flop_per_launch": flop, "ms_per_launch": gemm_ms},
            "kernels": {"acrl_lmhead_logits_stats": {"ms": gemm_ms, "TFLOP/s": tf},
                        "acrl_lmhead_merge": {"ms": merge_ms},
                        "acrl_loss_grad_logits": {"ms": grad_ms,
