@@ -19,7 +19,7 @@
 //              row), round to bf16, fold the statistics, and write the logits
 //              through shared memory with TMA bulk tensor stores (32 x 32
 //              blocks, two staging buffers per warp).
-// Tiles are visited in bands of 16 row tiles so that the weight tiles in
+// Tiles are visited in bands of 32 row tiles so that the weight tiles in
 // flight are shared through L2 by the clusters working on the same band.
 // Every wait on an mbarrier is bounded in time; on expiry the kernel raises
 // ACRL_FLAG_TIMEOUT, lets the copies it issued land, and exits after freeing
@@ -40,7 +40,7 @@ namespace {
 constexpr int kBM = 128, kBN = 256;
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
-constexpr int kBandM = 16;
+constexpr int kBandM = 32;
 // Output staging: each epilogue warp owns two 32 x 32 bf16 blocks (its 32
 // rows x one 32-column chunk of the accumulator), stored 64-byte-swizzled.
 constexpr int kOutBlockBytes = 32 * 32 * 2;
