@@ -40,9 +40,10 @@ def _check_logits(got_bf16, ref, abs_sum, K, what="logits"):
 
 
 # also: one row and a vocabulary narrower than a 32-column store block; an odd number of row tiles (the second
-# CTA of the last cluster has no rows) with a ragged K; K narrower than one 64-column slab
+# CTA of the last cluster has no rows) with a ragged K; K narrower than one 64-column slab; 66 row tiles, i.e.
+# three bands of row-tile pairs (16, 16 and a ragged 1) with a ragged last tile
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (200, 1000, 328), (384, 2304, 4096), (130, 151936, 64),
-                                   (1, 8, 64), (257, 520, 72), (5, 40, 8)])
+                                   (1, 8, 64), (257, 520, 72), (5, 40, 8), (8322, 1000, 64)])
 def test_lmhead_small_shapes(M, N, K):
     gen = torch.Generator(device=DEV).manual_seed(M * 7 + N + K)
     H = torch.randn((M, K), generator=gen, device=DEV).to(torch.bfloat16)
