@@ -215,6 +215,19 @@ def _bf16_rows_f64(O, t, rows, cols):
 _POOL = None
 
 
+def _cpu_model():
+    """The host CPU's model name (lscpu), or the machine type."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.machine()
+
+
 def _oracle_pool():
     """Worker processes for the oracle's row blocks, one per host core the
     process may run on (spawned, so they never inherit a CUDA context), all
@@ -360,7 +373,8 @@ def run_reference(args):
            "ms_per_step": float(np.median(t_all[args.warmup:])) * 1e3,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": config,
-           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
+                            "cpu": _cpu_model()},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
     return 0
@@ -553,7 +567,8 @@ def run_ours(args):
         out["e2e"] = e2e
     if not args.no_cpu and world == 1:
         v, desc, n, cores = oracle_tokens_per_s(batch, params, rows_budget_s=args.ref_seconds, max_rows=16384)
-        out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc}
+        out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
+                               "cpu": _cpu_model()}
     print(json.dumps(out))
     return 0
 
@@ -673,7 +688,8 @@ def run_lmhead(args):
            "clocks": clocks.summary(), "gpu_launches": 10 * args.steps}
     if not args.no_cpu:
         v, desc, _, cores = oracle_tokens_per_s(b, p, rows_budget_s=args.ref_seconds, lmhead=True)
-        out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc}
+        out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
+                               "cpu": _cpu_model()}
     print(json.dumps(out))
     return 0
 
