@@ -760,6 +760,18 @@ def _huge_empty(shape, dtype):
     return arr
 
 
+def _host_available_bytes():
+    """MemAvailable of the host (Linux), or None."""
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return None
+
+
 def run_e2e(batch, step, params, args, dev):
     """Same metric through the public API with the user's buffers in host
     memory: every step uploads that step's inputs from page-locked host memory,
@@ -773,7 +785,12 @@ def run_e2e(batch, step, params, args, dev):
     T, ld = batch.logits.shape
     V = batch.V
     # The user's host arrays, page-locked and of exactly their size (torch's pinned allocator would round 44.8 GB
-    # up to 64 GB).
+    # up to 64 GB).  Page-locking most of the host's memory could starve it, so leave a margin.
+    need = 2 * T * ld * 2
+    avail = _host_available_bytes()
+    if avail is not None and need + (32 << 30) > avail:
+        return {"value": None, "unit": UNIT,
+                "error": f"skipped: {need / 1e9:.1f} GB of page-locked buffers with {avail / 1e9:.1f} GB available"}
     pinned = _PinnedHost()
     try:
         try:
