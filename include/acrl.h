@@ -357,6 +357,54 @@ acrl_status acrl_loss_grad_logits(const acrl_bf16* logits, int64_t T, int64_t V,
 acrl_status acrl_reduce_loss(const float* token_loss, int64_t T, float* loss, acrl_stream stream);
 
 /*
+ * Host-buffer pipeline -- the whole on-policy pass (token statistics,
+ * discrepancy, advantages, controller, gradient: the calls above) for a batch
+ * whose inputs and outputs live in host memory, e.g. logits computed on or
+ * offloaded to the host.  Per step the logits are uploaded in `chunks` row
+ * chunks and the statistics call runs on each chunk as it lands; then the
+ * discrepancy, advantage and controller calls; then the gradient call chunk
+ * by chunk, each gradient chunk downloaded as soon as it is written, and the
+ * loss.  Uploads run on one copy stream of the pipeline and downloads on
+ * another, so consecutive steps overlap: step k+1's uploads run while step
+ * k's gradient is downloaded.  The results are those of the device calls on
+ * the same data, bit for bit.
+ *
+ * acrl_host_pipeline_workspace_bytes -- device bytes the pipeline needs: the
+ *   batch's logits [T, ld], a ring of up to four gradient chunks, the
+ *   per-token and per-response vectors and two copies of the small inputs.
+ * acrl_host_pipeline_create -- binds a caller-owned device workspace of at
+ *   least that size (16-byte aligned; the library allocates no device memory)
+ *   and creates the two copy streams and the events that order the chunks.
+ *   T >= 1, 1 <= V <= ld (ld a multiple of 8), S >= 1, Gn >= 1,
+ *   1 <= chunks <= 4096.  *pipeline receives the handle.
+ * acrl_host_pipeline_step -- enqueues one step.  Host arrays, page-locked for
+ *   the copies to overlap (ordinary memory works, without overlap):
+ *     logits bf16 [T, ld], ids int32 [T], mask uint8 [T] (or NULL: all 1),
+ *     logp_mu float [T], rewards float [S], seq_offsets int64 [S+1],
+ *     group_offsets int32 [Gn+1]  -- read while the uploads run;
+ *     grad bf16 [T, ld] (columns >= V untouched), loss float [1]
+ *                                 -- written while the downloads run.
+ *   `state` is the device controller state, `p` the parameters (with
+ *   p->entropy_coeff > 0 the entropy bonus is included), `dev_flags` the
+ *   device flags word.  The kernels run on `stream`, which is made to wait
+ *   for the step's downloads: once `stream` has been synchronised, grad and
+ *   loss hold the step's results.  Host arrays must stay valid until then.
+ *   One host thread at a time per pipeline.
+ * acrl_host_pipeline_destroy -- waits for the pipeline's copies, releases its
+ *   streams and events (not the workspace) and frees the handle.
+ */
+typedef struct acrl_host_pipeline acrl_host_pipeline;
+int64_t     acrl_host_pipeline_workspace_bytes(int64_t T, int64_t ld, int32_t S, int32_t Gn, int32_t chunks);
+acrl_status acrl_host_pipeline_create(acrl_host_pipeline** pipeline, int64_t T, int64_t V, int64_t ld, int32_t S,
+                                      int32_t Gn, int32_t chunks, void* workspace, int64_t workspace_bytes);
+acrl_status acrl_host_pipeline_step(acrl_host_pipeline* pipeline, const acrl_params* p,
+                                    acrl_controller_state* state, const acrl_bf16* logits, const int32_t* ids,
+                                    const uint8_t* mask, const float* logp_mu, const float* rewards,
+                                    const int64_t* seq_offsets, const int32_t* group_offsets, acrl_bf16* grad,
+                                    float* loss, int32_t* dev_flags, acrl_stream stream);
+acrl_status acrl_host_pipeline_destroy(acrl_host_pipeline* pipeline);
+
+/*
  * acrl_lmhead_logits_stats -- the LM-head projection logits = H W^T fused
  * with the log-softmax statistics of acrl_token_stats (the optional fused
  * path of the logits pass; the paper's policy pi ends in this projection).

@@ -73,6 +73,12 @@ SIGNATURES = {
     "acrl_loss_grad_logits": (c_i32, [c_p, c_i64, c_i64, c_i64, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_f32, c_p, c_p,
                                       c_p, c_p, c_p]),
     "acrl_reduce_loss": (c_i32, [c_p, c_i64, c_p, c_p]),
+    "acrl_host_pipeline_workspace_bytes": (c_i64, [c_i64, c_i64, c_i32, c_i32, c_i32]),
+    "acrl_host_pipeline_create": (c_i32, [ctypes.POINTER(c_p), c_i64, c_i64, c_i64, c_i32, c_i32, c_i32, c_p,
+                                          c_i64]),
+    "acrl_host_pipeline_step": (c_i32, [c_p, ctypes.POINTER(Params), c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p,
+                                        c_p, c_p, c_p]),
+    "acrl_host_pipeline_destroy": (c_i32, [c_p]),
     "acrl_lmhead_workspace_bytes": (c_i64, [c_i64, c_i64]),
     "acrl_lmhead_logits_stats": (c_i32, [c_p, c_i64, c_i64, c_i64, c_p, c_i64, c_i64, c_p, c_i64, c_p, c_p, c_p]),
     "acrl_lmhead_merge": (c_i32, [c_p, c_p, c_i64, c_i64, c_i64, c_p, c_p, c_p, c_p, c_p, c_p, c_p]),

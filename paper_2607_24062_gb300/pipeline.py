@@ -14,13 +14,14 @@ to a callback.
 
 from __future__ import annotations
 
+import ctypes
 from dataclasses import dataclass
 from typing import Callable
 
 import torch
 
 from . import api
-from ._abi import BATCH_DTYPE, GRP_DTYPE, SEQ_DTYPE, Params
+from ._abi import BATCH_DTYPE, GRP_DTYPE, SEQ_DTYPE, STATE_DTYPE, AcrlError, Params, check
 
 
 class AcrlStep:
@@ -167,3 +168,69 @@ def importance_weights(state, params: Params, logp_old, logp_mu, mask, rewards, 
     weight, coef, alpha = api.controller_step(state, params, disc, mask, seq_offsets, group_offsets, adv, flags=flags,
                                               stream=stream)
     return Weights(weight, coef, adv, alpha, disc, flags)
+
+
+def _host(t, dtype, n, name):
+    if not isinstance(t, torch.Tensor) or t.device.type != "cpu":
+        raise AcrlError(f"{name}: expected a host (CPU) tensor")
+    if t.dtype != dtype or not t.is_contiguous() or t.numel() < n:
+        raise AcrlError(f"{name}: expected a contiguous {dtype} tensor of at least {n} elements")
+    return t.data_ptr()
+
+
+class HostPipeline:
+    """acrl_host_pipeline_*: the whole on-policy pass for batches whose inputs
+    and outputs are host tensors (page-locked for the copies to overlap),
+    with the batch shape (T, V, ld, S, Gn) fixed at construction.  Uploads,
+    the five calls and the downloads run chunk by chunk on the library's own
+    streams; consecutive steps overlap.  `step` only enqueues: the host
+    gradient and loss are valid once `stream` (default: the current stream)
+    has been synchronised."""
+
+    def __init__(self, T: int, V: int, ld: int, S: int, Gn: int, chunks: int = 16, device="cuda"):
+        L = api.lib()
+        nbytes = L.acrl_host_pipeline_workspace_bytes(T, ld, S, Gn, chunks)
+        if nbytes < 0:
+            raise AcrlError("acrl_host_pipeline_workspace_bytes: invalid shape")
+        dev = torch.device(device)
+        self.device = torch.device("cuda", torch.cuda.current_device()) if dev.index is None else dev
+        self.T, self.V, self.ld, self.S, self.Gn, self.chunks = T, V, ld, S, Gn, chunks
+        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=self.device)
+        self.handle = ctypes.c_void_p()
+        with torch.cuda.device(self.device):
+            check(L.acrl_host_pipeline_create(ctypes.byref(self.handle), T, V, ld, S, Gn, chunks,
+                                              self.workspace.data_ptr(), nbytes), "acrl_host_pipeline_create")
+
+    def step(self, state: torch.Tensor, params: Params, logits, ids, mask, logp_mu, rewards, seq_offsets,
+             group_offsets, grad, loss, flags: torch.Tensor, stream=None) -> None:
+        if not self.handle:
+            raise AcrlError("host pipeline: already closed")
+        T, ld, S, Gn = self.T, self.ld, self.S, self.Gn
+        if logits.dim() != 2 or logits.shape[0] != T or logits.stride(0) != ld or grad.dim() != 2 or \
+                grad.shape[0] != T or grad.stride(0) != ld:
+            raise AcrlError(f"logits / grad: expected host bf16 [{T}, {ld}] tensors")
+        ptrs = (_host(logits, torch.bfloat16, T * ld, "logits"), _host(ids, torch.int32, T, "ids"),
+                None if mask is None else _host(mask, torch.uint8, T, "mask"),
+                _host(logp_mu, torch.float32, T, "logp_mu"), _host(rewards, torch.float32, S, "rewards"),
+                _host(seq_offsets, torch.int64, S + 1, "seq_offsets"),
+                _host(group_offsets, torch.int32, Gn + 1, "group_offsets"),
+                _host(grad, torch.bfloat16, T * ld, "grad"), _host(loss, torch.float32, 1, "loss"))
+        api._need(state, torch.uint8, STATE_DTYPE.itemsize, "state")
+        api._need(flags, torch.int32, 1, "flags")
+        if state.device != self.device or flags.device != self.device:
+            raise AcrlError("state / flags: expected on the pipeline's device")
+        with torch.cuda.device(self.device):
+            s = torch.cuda.current_stream(self.device) if stream is None else stream
+            check(api.lib().acrl_host_pipeline_step(self.handle, ctypes.byref(params), state.data_ptr(), *ptrs,
+                                                    flags.data_ptr(), s.cuda_stream), "acrl_host_pipeline_step")
+
+    def close(self) -> None:
+        if self.handle:
+            h, self.handle = self.handle, ctypes.c_void_p()
+            check(api.lib().acrl_host_pipeline_destroy(h), "acrl_host_pipeline_destroy")
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

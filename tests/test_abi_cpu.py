@@ -73,6 +73,21 @@ def test_host_side_rejections(L):
     assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(x_ema=1.5)), None) == E
     assert L.acrl_controller_init(fake, ctypes.byref(_abi.Params(entropy_coeff=-1.0)), None) == E
     assert L.acrl_read_flags(None, None, None) == E
+    # the host-buffer pipeline: shapes, workspace and handle checked before any CUDA call
+    assert L.acrl_host_pipeline_workspace_bytes(0, 16, 1, 1, 1) == -1
+    assert L.acrl_host_pipeline_workspace_bytes(4, 16, 1, 1, 5000) == -1
+    ws = L.acrl_host_pipeline_workspace_bytes(64, 16, 2, 1, 4)
+    assert ws > 64 * 16 * 2
+    h = ctypes.c_void_p()
+    assert L.acrl_host_pipeline_create(None, 64, 16, 16, 2, 1, 4, fake, ws) == E
+    assert L.acrl_host_pipeline_create(ctypes.byref(h), 64, 16, 12, 2, 1, 4, fake, ws) == E       # ld < V
+    assert L.acrl_host_pipeline_create(ctypes.byref(h), 3, 16, 16, 2, 1, 4, fake, ws) == E        # chunks > T
+    assert L.acrl_host_pipeline_create(ctypes.byref(h), 64, 16, 16, 2, 1, 4, fake, ws - 1) == E   # too small
+    assert L.acrl_host_pipeline_create(ctypes.byref(h), 64, 16, 16, 2, 1, 4, fake + 8, ws) == E   # misaligned
+    assert h.value is None
+    assert L.acrl_host_pipeline_step(None, ctypes.byref(p), fake, fake, fake, None, fake, fake, fake, fake, fake,
+                                     fake, fake, None) == E
+    assert L.acrl_host_pipeline_destroy(None) == E
     assert L.acrl_controller_save(None, fake, None) == E and L.acrl_controller_save(fake, None, None) == E
     assert L.acrl_controller_load(None, fake, None) == E and L.acrl_controller_load(fake, None, None) == E
     assert L.acrl_reduce_loss(None, 4, fake, None) == E
