@@ -773,12 +773,11 @@ def _host_available_bytes():
 
 
 def run_e2e(batch, step, params, args, dev):
-    """Same metric through the public API with the user's buffers in host
-    memory: every step uploads that step's inputs from page-locked host memory,
-    runs the whole path and downloads the gradient and the loss.  Rows move in
-    chunks on a copy stream so that uploads overlap the statistics kernel and
-    downloads overlap the gradient kernel; events order every reuse of a
-    device or host chunk."""
+    """Same metric through the C ABI with the user's buffers in host memory:
+    one acrl_host_pipeline_step call per step, which uploads that step's
+    inputs from page-locked host memory in row chunks, runs the whole path and
+    downloads the gradient and the loss chunk by chunk on the library's own
+    copy streams (consecutive steps overlap)."""
     import torch
 
     import paper_2607_24062_gb300 as acrl
@@ -792,6 +791,7 @@ def run_e2e(batch, step, params, args, dev):
         return {"value": None, "unit": UNIT,
                 "error": f"skipped: {need / 1e9:.1f} GB of page-locked buffers with {avail / 1e9:.1f} GB available"}
     pinned = _PinnedHost()
+    hp = None
     try:
         try:
             h_logits_np = pinned.empty((T, ld), np.uint16)
@@ -803,70 +803,14 @@ def run_e2e(batch, step, params, args, dev):
         h_logits.copy_(batch.logits)
         small_h = {k: getattr(batch, k).cpu().pin_memory()
                    for k in ("ids", "mask", "logp_mu", "rewards", "seq_offsets", "group_offsets")}
-        # two device copies of the O(T) inputs, alternating by step parity
-        small_d = [{k: torch.empty_like(v, device=dev) for k, v in small_h.items()} for _ in range(2)]
         loss_h = torch.empty(1, dtype=torch.float32, pin_memory=True)
-        d_logits = batch.logits
-        comp = torch.cuda.current_stream(dev)
-        # One copy stream per direction: the next step's uploads run while this step's gradient downloads,
-        # which moves more bytes per second over the host link than either direction alone.
-        s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
         nchunk = max(1, args.e2e_chunks)
-        bounds = [(T * k // nchunk, T * (k + 1) // nchunk) for k in range(nchunk)]
-        E = torch.cuda.Event
-        ev_up = [E() for _ in bounds]      # chunk uploaded
-        ev_used = [E() for _ in bounds]    # gradient kernel done reading the chunk's logits
-        ev_grad = [E() for _ in bounds]    # gradient chunk written
-        ev_down = [E() for _ in bounds]    # gradient chunk downloaded
-        ev_small = [E(), E()]
-        ev_done = [E(), E()]               # all of a step's kernels done (by parity)
-        ev_loss = E()
-        count = [0]
+        hp = acrl.HostPipeline(T, V, ld, batch.S, batch.Gn, chunks=nchunk, device=dev)
+        comp = torch.cuda.current_stream(dev)
 
         def one():
-            k = count[0]
-            par = k & 1
-            sd = small_d[par]
-            with torch.cuda.stream(s_in):
-                if k >= 2:
-                    s_in.wait_event(ev_done[par])
-                for name, v in small_h.items():
-                    sd[name].copy_(v, non_blocking=True)
-                ev_small[par].record(s_in)
-                for c, (r0, r1) in enumerate(bounds):
-                    if k >= 1:
-                        s_in.wait_event(ev_used[c])
-                    d_logits[r0:r1].copy_(h_logits[r0:r1], non_blocking=True)
-                    ev_up[c].record(s_in)
-            comp.wait_event(ev_small[par])
-            for c, (r0, r1) in enumerate(bounds):
-                comp.wait_event(ev_up[c])
-                acrl.token_stats(d_logits[r0:r1], sd["ids"][r0:r1], sd["mask"][r0:r1], V=V, lse=step.lse[r0:r1],
-                                 logp=step.logp[r0:r1], entropy=step.entropy[r0:r1], flags=step.flags)
-            acrl.seq_discrepancy(step.logp, sd["logp_mu"], sd["mask"], sd["seq_offsets"], sd["group_offsets"],
-                                 step.entropy, out=step.disc, flags=step.flags)
-            acrl.grpo_advantage(sd["rewards"], sd["group_offsets"], params, adv=step.adv, flags=step.flags)
-            acrl.controller_step(step.state, params, step.disc, sd["mask"], sd["seq_offsets"], sd["group_offsets"],
-                                 step.adv, weight=step.weight, coef=step.coef, alpha=step.alpha, flags=step.flags)
-            for c, (r0, r1) in enumerate(bounds):
-                if k >= 1:
-                    comp.wait_event(ev_down[c])
-                acrl.loss_grad_logits(d_logits[r0:r1], sd["ids"][r0:r1], sd["mask"][r0:r1], step.lse[r0:r1], None,
-                                      step.coef[r0:r1], params.clip_eps, V=V, grad=step.grad[r0:r1],
-                                      token_loss=step.token_loss[r0:r1], loss=step.chunk_loss, flags=step.flags)
-                ev_used[c].record(comp)
-                ev_grad[c].record(comp)
-                with torch.cuda.stream(s_out):
-                    s_out.wait_event(ev_grad[c])
-                    h_grad[r0:r1].copy_(step.grad[r0:r1], non_blocking=True)
-                    ev_down[c].record(s_out)
-            acrl.reduce_loss(step.token_loss, loss=step.loss)
-            ev_loss.record(comp)
-            ev_done[par].record(comp)
-            with torch.cuda.stream(s_out):
-                s_out.wait_event(ev_loss)
-                loss_h.copy_(step.loss, non_blocking=True)
-            count[0] += 1
+            hp.step(step.state, params, h_logits, small_h["ids"], small_h["mask"], small_h["logp_mu"],
+                    small_h["rewards"], small_h["seq_offsets"], small_h["group_offsets"], h_grad, loss_h, step.flags)
 
         one()
         torch.cuda.synchronize()
@@ -875,8 +819,7 @@ def run_e2e(batch, step, params, args, dev):
         t0.record(comp)
         for _ in range(n):
             one()
-        comp.wait_stream(s_out)   # the last step's gradient and loss are on the host
-        t1.record(comp)
+        t1.record(comp)            # the pipeline makes this stream wait for each step's downloads
         torch.cuda.synchronize()
         ms = t0.elapsed_time(t1) / n
         ok = bool(torch.equal(h_grad[:, :V].view(torch.int16)[:: max(1, T // 64)].to(dev),
@@ -886,8 +829,10 @@ def run_e2e(batch, step, params, args, dev):
         return {"value": int(batch.mask.sum()) / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n, "chunks": nchunk,
                 "host_link_GB/s": (h2d + d2h) / (ms / 1e3) / 1e9, "download_matches_device": ok,
-                "host_memory": pinned.describe()}
+                "api": "acrl_host_pipeline_step (C ABI), host buffers", "host_memory": pinned.describe()}
     finally:
+        if hp is not None:
+            hp.close()
         pinned.free()
 
 
