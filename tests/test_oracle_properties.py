@@ -16,7 +16,8 @@ from hypothesis import strategies as st  # noqa: E402
 
 import oracle as O  # noqa: E402
 
-SETTINGS = settings(max_examples=60, deadline=None)
+# derandomized: the same examples every run, so that the suite's outcome does not depend on the run
+SETTINGS = settings(max_examples=60, deadline=None, derandomize=True)
 
 
 @st.composite
