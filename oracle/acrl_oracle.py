@@ -313,10 +313,13 @@ def grpo_advantage(rewards, group_offsets, params: Params):
         if G == 1:
             A[go[g]] = r[0] if params.singleton_rule == SINGLETON_MEAN0_STD1 else 0.0
             continue
+        if np.all(r == r[0]):
+            # equal rewards: every R_i - mean is exactly 0, so A = 0 (0/0 read as 0 when adv_eps = 0); decided
+            # here exactly, since a float64 mean of values with full 53-bit significands can miss them by an ulp
+            continue
         mean = r.sum() / G
         var = ((r - mean) ** 2).sum() / (G - params.adv_ddof) if G > params.adv_ddof else 0.0
         den = math.sqrt(var) + params.adv_eps
-        # equal rewards with adv_eps = 0 give 0/0: such a prompt carries no advantage, A = 0
         A[go[g]:go[g + 1]] = (r - mean) / den if den > 0 else 0.0
     return A
 

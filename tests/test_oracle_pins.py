@@ -211,6 +211,11 @@ def test_grpo_equal_rewards_without_epsilon():
     A = O.grpo_advantage(np.array([1.0, 1.0, 1.0, 0.0, 1.0]), [0, 3, 5], O.Params(adv_eps=0.0))
     assert np.all(A[:3] == 0.0)
     np.testing.assert_allclose(A[3:], [-math.sqrt(0.5), math.sqrt(0.5)], rtol=1e-14)   # (0 or 1 - 0.5) / sqrt(0.5)
+    # equal rewards whose float64 mean is not exact (found by the property test): still no advantage
+    r = 0.9798852880475015
+    assert sum([r, r, r]) / 3 != r
+    for eps in (0.0, 1e-6):
+        assert np.all(O.grpo_advantage(np.array([r, r, r]), [0, 3], O.Params(adv_eps=eps)) == 0.0)
 
 
 def test_grpo_special_groups():
