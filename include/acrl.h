@@ -12,8 +12,10 @@
  * Conventions shared by every call:
  *   - Pointers documented "device" must be device memory of the current CUDA
  *     device (or managed memory).  The caller owns every buffer; the library
- *     allocates nothing and keeps no global state, except the fixed scratch
- *     array of acrl_lmhead_stats_noalloc (documented there).
+ *     allocates no device memory and keeps no global state, except the fixed
+ *     scratch array of acrl_lmhead_stats_noalloc (documented there).  The
+ *     host-buffer pipeline's handle owns two streams and its events, made by
+ *     acrl_host_pipeline_create and released by acrl_host_pipeline_destroy.
  *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL is the
  *     legacy default stream) except acrl_read_flags and acrl_check_flags,
  *     which synchronise it.
