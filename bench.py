@@ -528,7 +528,10 @@ def run_ours(args):
         e2e = run_e2e(batch, step, params, args, dev)
         if world > 1 and e2e is not None:
             e2e["ranks_measured"] = 1
-            e2e["note"] = "rank 0 alone, the other ranks idle: one GPU's host link, not the whole job"
+            e2e["note"] = ("rank 0 alone, the other ranks idle: one GPU's host link, not the whole job; the host "
+                           "pipeline has no rank exchange, so its weights use rank 0's batch statistics and its "
+                           "gradient is not compared with the exchanged step's")
+            e2e["download_matches_device"] = None
     if world > 1:
         dist.barrier()
     if rank != 0:
