@@ -392,6 +392,17 @@ acrl_status acrl_reduce_loss(const float* token_loss, int64_t T, float* loss, ac
  *   for the step's downloads: once `stream` has been synchronised, grad and
  *   loss hold the step's results.  Host arrays must stay valid until then.
  *   One host thread at a time per pipeline.
+ * acrl_host_pipeline_begin / acrl_host_pipeline_finish -- the same step in
+ *   two halves, for data-parallel callers: begin enqueues the uploads, the
+ *   statistics and the discrepancy call (the arguments the step reads from
+ *   host memory, plus dev_flags and stream); then the caller may combine the
+ *   batch statistics across ranks on `stream` (n_tokens, n_groups_valid and
+ *   Y_sum of the acrl_batch_stats at acrl_host_pipeline_batch_stats, as for
+ *   acrl_controller_step); finish enqueues the advantages, the controller, the
+ *   gradient, the downloads and the loss.  step = begin + finish.  Calls out
+ *   of that order return ACRL_ERR_INVALID_ARG.
+ * acrl_host_pipeline_batch_stats -- device address of the pipeline's
+ *   acrl_batch_stats (inside the workspace), or NULL for a NULL handle.
  * acrl_host_pipeline_destroy -- waits for the pipeline's copies, releases its
  *   streams and events (not the workspace) and frees the handle.
  */
@@ -404,6 +415,14 @@ acrl_status acrl_host_pipeline_step(acrl_host_pipeline* pipeline, const acrl_par
                                     const uint8_t* mask, const float* logp_mu, const float* rewards,
                                     const int64_t* seq_offsets, const int32_t* group_offsets, acrl_bf16* grad,
                                     float* loss, int32_t* dev_flags, acrl_stream stream);
+acrl_status acrl_host_pipeline_begin(acrl_host_pipeline* pipeline, const acrl_bf16* logits, const int32_t* ids,
+                                     const uint8_t* mask, const float* logp_mu, const float* rewards,
+                                     const int64_t* seq_offsets, const int32_t* group_offsets, int32_t* dev_flags,
+                                     acrl_stream stream);
+acrl_status acrl_host_pipeline_finish(acrl_host_pipeline* pipeline, const acrl_params* p,
+                                      acrl_controller_state* state, acrl_bf16* grad, float* loss,
+                                      int32_t* dev_flags, acrl_stream stream);
+acrl_batch_stats* acrl_host_pipeline_batch_stats(acrl_host_pipeline* pipeline);
 acrl_status acrl_host_pipeline_destroy(acrl_host_pipeline* pipeline);
 
 /*

@@ -78,6 +78,9 @@ SIGNATURES = {
                                           c_i64]),
     "acrl_host_pipeline_step": (c_i32, [c_p, ctypes.POINTER(Params), c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p,
                                         c_p, c_p, c_p]),
+    "acrl_host_pipeline_begin": (c_i32, [c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p, c_p]),
+    "acrl_host_pipeline_finish": (c_i32, [c_p, ctypes.POINTER(Params), c_p, c_p, c_p, c_p, c_p]),
+    "acrl_host_pipeline_batch_stats": (c_p, [c_p]),
     "acrl_host_pipeline_destroy": (c_i32, [c_p]),
     "acrl_lmhead_workspace_bytes": (c_i64, [c_i64, c_i64]),
     "acrl_lmhead_logits_stats": (c_i32, [c_p, c_i64, c_i64, c_i64, c_p, c_i64, c_i64, c_p, c_i64, c_p, c_p, c_p]),

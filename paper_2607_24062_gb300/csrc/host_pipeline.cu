@@ -85,6 +85,8 @@ struct acrl_host_pipeline {
     int64_t T, V, ld;
     int32_t S, Gn, chunks, ring;
     int64_t step;
+    bool begun;      // begin enqueued, finish not yet
+    bool has_mask;   // the begun step's mask was given
     char* ws;
     Layout L;
     cudaStream_t up, down;
@@ -161,14 +163,11 @@ extern "C" acrl_status acrl_host_pipeline_create(acrl_host_pipeline** pipeline, 
     return ACRL_OK;
 }
 
-extern "C" acrl_status acrl_host_pipeline_step(acrl_host_pipeline* pl, const acrl_params* p,
-                                               acrl_controller_state* state, const acrl_bf16* logits,
-                                               const int32_t* ids, const uint8_t* mask, const float* logp_mu,
-                                               const float* rewards, const int64_t* seq_offsets,
-                                               const int32_t* group_offsets, acrl_bf16* grad, float* loss,
-                                               int32_t* dev_flags, acrl_stream stream) {
-    if (!pl || !params_ok(p) || !state || !logits || !ids || !logp_mu || !rewards || !seq_offsets ||
-        !group_offsets || !grad || !loss || !dev_flags)
+extern "C" acrl_status acrl_host_pipeline_begin(acrl_host_pipeline* pl, const acrl_bf16* logits, const int32_t* ids,
+                                                const uint8_t* mask, const float* logp_mu, const float* rewards,
+                                                const int64_t* seq_offsets, const int32_t* group_offsets,
+                                                int32_t* dev_flags, acrl_stream stream) {
+    if (!pl || pl->begun || !logits || !ids || !logp_mu || !rewards || !seq_offsets || !group_offsets || !dev_flags)
         return ACRL_ERR_INVALID_ARG;
     cudaStream_t comp = reinterpret_cast<cudaStream_t>(stream);
     const Layout& L = pl->L;
@@ -180,7 +179,6 @@ extern "C" acrl_status acrl_host_pipeline_step(acrl_host_pipeline* pl, const acr
     int32_t* d_ids = pl->at<int32_t>(L.ids[slot]);
     uint8_t* d_mask = mask ? pl->at<uint8_t>(L.mask[slot]) : nullptr;
     float* d_mu = pl->at<float>(L.mu[slot]);
-    float* d_rewards = pl->at<float>(L.rewards[slot]);
     int64_t* d_so = pl->at<int64_t>(L.so[slot]);
     int32_t* d_go = pl->at<int32_t>(L.go[slot]);
     acrl_bf16* d_logits = pl->at<acrl_bf16>(L.logits);
@@ -188,7 +186,8 @@ extern "C" acrl_status acrl_host_pipeline_step(acrl_host_pipeline* pl, const acr
         !ok(cudaMemcpyAsync(d_ids, ids, T * 4, cudaMemcpyHostToDevice, pl->up)) ||
         (mask && !ok(cudaMemcpyAsync(d_mask, mask, T, cudaMemcpyHostToDevice, pl->up))) ||
         !ok(cudaMemcpyAsync(d_mu, logp_mu, T * 4, cudaMemcpyHostToDevice, pl->up)) ||
-        !ok(cudaMemcpyAsync(d_rewards, rewards, int64_t(S) * 4, cudaMemcpyHostToDevice, pl->up)) ||
+        !ok(cudaMemcpyAsync(pl->at<float>(L.rewards[slot]), rewards, int64_t(S) * 4, cudaMemcpyHostToDevice,
+                            pl->up)) ||
         !ok(cudaMemcpyAsync(d_so, seq_offsets, (int64_t(S) + 1) * 8, cudaMemcpyHostToDevice, pl->up)) ||
         !ok(cudaMemcpyAsync(d_go, group_offsets, (int64_t(Gn) + 1) * 4, cudaMemcpyHostToDevice, pl->up)) ||
         !ok(cudaEventRecord(pl->ev_small()[slot], pl->up)))
@@ -202,7 +201,7 @@ extern "C" acrl_status acrl_host_pipeline_step(acrl_host_pipeline* pl, const acr
             return ACRL_ERR_CUDA;
     }
 
-    // statistics, chunk by chunk as the logits land
+    // statistics, chunk by chunk as the logits land, then the discrepancy call
     float* lse = pl->at<float>(L.lse);
     float* logp = pl->at<float>(L.logp);
     float* ent = pl->at<float>(L.ent);
@@ -215,21 +214,45 @@ extern "C" acrl_status acrl_host_pipeline_step(acrl_host_pipeline* pl, const acr
                                                 dev_flags, stream);
         if (st != ACRL_OK) return st;
     }
+    const acrl_status st = acrl_seq_discrepancy(logp, d_mu, d_mask, T, d_so, S, d_go, Gn, ent, pl->at<float>(L.lr),
+                                                pl->at<float>(L.d), pl->at<acrl_seq_stats>(L.seq),
+                                                pl->at<acrl_group_stats>(L.grp), pl->at<acrl_batch_stats>(L.batch),
+                                                dev_flags, stream);
+    if (st != ACRL_OK) return st;
+    pl->begun = true;
+    pl->has_mask = mask != nullptr;
+    return ACRL_OK;
+}
 
-    // discrepancy, advantages, controller
+extern "C" acrl_status acrl_host_pipeline_finish(acrl_host_pipeline* pl, const acrl_params* p,
+                                                 acrl_controller_state* state, acrl_bf16* grad, float* loss,
+                                                 int32_t* dev_flags, acrl_stream stream) {
+    if (!pl || !pl->begun || !params_ok(p) || !state || !grad || !loss || !dev_flags) return ACRL_ERR_INVALID_ARG;
+    pl->begun = false;
+    cudaStream_t comp = reinterpret_cast<cudaStream_t>(stream);
+    const Layout& L = pl->L;
+    const int64_t T = pl->T, ld = pl->ld, row_bytes = ld * 2;
+    const int S = pl->S, Gn = pl->Gn, C = pl->chunks, slot = int(pl->step & 1);
+    pl->step += 1;
+    auto ok = [](cudaError_t e) { return e == cudaSuccess; };
+    int32_t* d_ids = pl->at<int32_t>(L.ids[slot]);
+    uint8_t* d_mask = pl->has_mask ? pl->at<uint8_t>(L.mask[slot]) : nullptr;
+    int64_t* d_so = pl->at<int64_t>(L.so[slot]);
+    int32_t* d_go = pl->at<int32_t>(L.go[slot]);
+    acrl_bf16* d_logits = pl->at<acrl_bf16>(L.logits);
+    float* lse = pl->at<float>(L.lse);
+    float* ent = pl->at<float>(L.ent);
+
+    // advantages and controller
     acrl_seq_stats* seq = pl->at<acrl_seq_stats>(L.seq);
-    acrl_group_stats* grp = pl->at<acrl_group_stats>(L.grp);
-    acrl_batch_stats* batch = pl->at<acrl_batch_stats>(L.batch);
     float* adv = pl->at<float>(L.adv);
     float* coef = pl->at<float>(L.coef);
     float* ent_coef = p->entropy_coeff > 0.f ? pl->at<float>(L.ent_coef) : nullptr;
-    acrl_status st = acrl_seq_discrepancy(logp, d_mu, d_mask, T, d_so, S, d_go, Gn, ent, pl->at<float>(L.lr),
-                                          pl->at<float>(L.d), seq, grp, batch, dev_flags, stream);
-    if (st == ACRL_OK) st = acrl_grpo_advantage(d_rewards, d_go, Gn, S, p, adv, dev_flags, stream);
+    acrl_status st = acrl_grpo_advantage(pl->at<float>(L.rewards[slot]), d_go, Gn, S, p, adv, dev_flags, stream);
     if (st == ACRL_OK)
-        st = acrl_controller_step(state, p, pl->at<float>(L.lr), d_mask, T, d_so, S, d_go, Gn, seq, grp, batch, adv,
-                                  pl->at<float>(L.weight), coef, pl->at<float>(L.alpha), ent_coef, dev_flags,
-                                  stream);
+        st = acrl_controller_step(state, p, pl->at<float>(L.lr), d_mask, T, d_so, S, d_go, Gn, seq,
+                                  pl->at<acrl_group_stats>(L.grp), pl->at<acrl_batch_stats>(L.batch), adv,
+                                  pl->at<float>(L.weight), coef, pl->at<float>(L.alpha), ent_coef, dev_flags, stream);
     if (st != ACRL_OK) return st;
 
     // gradient, chunk by chunk into the ring, each chunk downloaded as soon as it is written
@@ -261,8 +284,24 @@ extern "C" acrl_status acrl_host_pipeline_step(acrl_host_pipeline* pl, const acr
         !ok(cudaEventRecord(pl->ev_fin(), pl->down)) || !ok(cudaStreamWaitEvent(comp, pl->ev_fin(), 0)) ||
         !ok(cudaEventRecord(pl->ev_done()[slot], comp)))
         return ACRL_ERR_CUDA;
-    pl->step += 1;
     return ACRL_OK;
+}
+
+extern "C" acrl_status acrl_host_pipeline_step(acrl_host_pipeline* pl, const acrl_params* p,
+                                               acrl_controller_state* state, const acrl_bf16* logits,
+                                               const int32_t* ids, const uint8_t* mask, const float* logp_mu,
+                                               const float* rewards, const int64_t* seq_offsets,
+                                               const int32_t* group_offsets, acrl_bf16* grad, float* loss,
+                                               int32_t* dev_flags, acrl_stream stream) {
+    if (!pl || pl->begun || !params_ok(p) || !state || !grad || !loss) return ACRL_ERR_INVALID_ARG;
+    const acrl_status st =
+        acrl_host_pipeline_begin(pl, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, dev_flags, stream);
+    if (st != ACRL_OK) return st;
+    return acrl_host_pipeline_finish(pl, p, state, grad, loss, dev_flags, stream);
+}
+
+extern "C" acrl_batch_stats* acrl_host_pipeline_batch_stats(acrl_host_pipeline* pl) {
+    return pl ? pl->at<acrl_batch_stats>(pl->L.batch) : nullptr;
 }
 
 extern "C" acrl_status acrl_host_pipeline_destroy(acrl_host_pipeline* pl) {

@@ -201,8 +201,19 @@ class HostPipeline:
             check(L.acrl_host_pipeline_create(ctypes.byref(self.handle), T, V, ld, S, Gn, chunks,
                                               self.workspace.data_ptr(), nbytes), "acrl_host_pipeline_create")
 
+    def batch_stats(self) -> torch.Tensor:
+        """The device bytes of the pipeline's acrl_batch_stats (a view into the workspace)."""
+        addr = api.lib().acrl_host_pipeline_batch_stats(self.handle)
+        off = addr - self.workspace.data_ptr()
+        return self.workspace[off: off + BATCH_DTYPE.itemsize]
+
     def step(self, state: torch.Tensor, params: Params, logits, ids, mask, logp_mu, rewards, seq_offsets,
-             group_offsets, grad, loss, flags: torch.Tensor, stream=None) -> None:
+             group_offsets, grad, loss, flags: torch.Tensor, stream=None,
+             exchange: Callable[[torch.Tensor], None] | None = None) -> None:
+        """One step; with `exchange` (e.g. distributed.allreduce_batch_stats) the
+        batch-statistics bytes are combined across ranks between the
+        discrepancy call and the controller (acrl_host_pipeline_begin, the
+        exchange on the stream, acrl_host_pipeline_finish)."""
         if not self.handle:
             raise AcrlError("host pipeline: already closed")
         T, ld, S, Gn = self.T, self.ld, self.S, self.Gn
@@ -219,10 +230,19 @@ class HostPipeline:
         api._need(flags, torch.int32, 1, "flags")
         if state.device != self.device or flags.device != self.device:
             raise AcrlError("state / flags: expected on the pipeline's device")
+        L = api.lib()
         with torch.cuda.device(self.device):
             s = torch.cuda.current_stream(self.device) if stream is None else stream
-            check(api.lib().acrl_host_pipeline_step(self.handle, ctypes.byref(params), state.data_ptr(), *ptrs,
-                                                    flags.data_ptr(), s.cuda_stream), "acrl_host_pipeline_step")
+            if exchange is None:
+                check(L.acrl_host_pipeline_step(self.handle, ctypes.byref(params), state.data_ptr(), *ptrs,
+                                                flags.data_ptr(), s.cuda_stream), "acrl_host_pipeline_step")
+                return
+            check(L.acrl_host_pipeline_begin(self.handle, *ptrs[:7], flags.data_ptr(), s.cuda_stream),
+                  "acrl_host_pipeline_begin")
+            with torch.cuda.stream(s):
+                exchange(self.batch_stats())
+            check(L.acrl_host_pipeline_finish(self.handle, ctypes.byref(params), state.data_ptr(), ptrs[7], ptrs[8],
+                                              flags.data_ptr(), s.cuda_stream), "acrl_host_pipeline_finish")
 
     def close(self) -> None:
         if self.handle:

@@ -88,6 +88,9 @@ def test_host_side_rejections(L):
     assert L.acrl_host_pipeline_step(None, ctypes.byref(p), fake, fake, fake, None, fake, fake, fake, fake, fake,
                                      fake, fake, None) == E
     assert L.acrl_host_pipeline_destroy(None) == E
+    assert L.acrl_host_pipeline_begin(None, fake, fake, None, fake, fake, fake, fake, fake, None) == E
+    assert L.acrl_host_pipeline_finish(None, ctypes.byref(p), fake, fake, fake, fake, None) == E
+    assert L.acrl_host_pipeline_batch_stats(None) is None
     assert L.acrl_controller_save(None, fake, None) == E and L.acrl_controller_save(fake, None, None) == E
     assert L.acrl_controller_load(None, fake, None) == E and L.acrl_controller_load(fake, None, None) == E
     assert L.acrl_reduce_loss(None, 4, fake, None) == E

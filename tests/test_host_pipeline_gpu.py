@@ -81,3 +81,38 @@ def test_host_pipeline_rejects_device_tensors_and_wrong_shapes():
         hp.step(state, p, b.logits.cpu(), b.ids.cpu(), None, b.logp_mu.cpu(), b.rewards.cpu(), b.seq_offsets.cpu(),
                 b.group_offsets.cpu(), grad, loss, flags)
     assert np.isfinite(float(loss[0]))
+
+
+def test_host_pipeline_exchange_matches_device_calls():
+    """The two-phase step (begin, the batch-statistics exchange, finish) with an
+    exchange that doubles the three summed fields, as an all-reduce over two
+    ranks holding the same batch would: the same results as AcrlStep with the
+    same exchange, bit for bit, over two steps."""
+    from paper_2607_24062_gb300 import distributed as D
+
+    def as_two_ranks(buf):
+        for name, dt in (("n_tokens", torch.int64), ("n_groups_valid", torch.int32), ("Y_sum", torch.float64)):
+            D._field(buf, name, dt).mul_(2)
+
+    spec = W.small_variant(W.GRPO, name="hp_x", n_prompts=3, group_size=4, len_lo=20, len_hi=120, V=3000,
+                           perturb_frac=0.4, perturb_std=0.3)
+    b = W.generate(spec, seed=43, device=DEV)
+    p = acrl.Params()
+    ref = acrl.AcrlStep.for_batch(b, p)
+    hp = acrl.HostPipeline(b.T, b.V, b.ld, b.S, b.Gn, chunks=5)
+    state, flags = api.controller_init(p), api.new_flags()
+    h = {k: _pinned(getattr(b, k)) for k in ("logits", "ids", "mask", "logp_mu", "rewards", "seq_offsets",
+                                             "group_offsets")}
+    for k in range(2):
+        grad = torch.zeros((b.T, b.ld), dtype=torch.bfloat16, pin_memory=True)
+        loss = torch.zeros(1, dtype=torch.float32, pin_memory=True)
+        hp.step(state, p, h["logits"], h["ids"], h["mask"], h["logp_mu"], h["rewards"], h["seq_offsets"],
+                h["group_offsets"], grad, loss, flags, exchange=as_two_ranks)
+        ref.run_batch(b, exchange=as_two_ranks)
+        torch.cuda.synchronize()
+        assert torch.equal(grad[:, : b.V].view(torch.int16), ref.grad[:, : b.V].cpu().view(torch.int16)), k
+        assert float(loss[0]) == float(ref.loss[0])
+        bs = api.read_structs(hp.batch_stats(), acrl.api.BATCH_DTYPE, 1)[0]
+        assert int(bs["n_groups_valid"]) == 2 * b.Gn
+    assert api.save_state(state) == api.save_state(ref.state)
+    hp.close()
