@@ -51,3 +51,13 @@ def test_c_client_whole_chain(tmp_path):
                    libs=(f"-L{cuda}/lib64", "-lcudart", f"-Wl,-rpath,{cuda}/lib64"))
     r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
     assert r.returncode == 0 and r.stdout.strip() == "ok", r.stdout + r.stderr
+
+
+@pytest.mark.gpu
+def test_c_client_host_pipeline(tmp_path):
+    """The host-buffer pipeline from C, bitwise against the device calls."""
+    cuda = os.environ.get("CUDA_HOME", "/usr/local/cuda")
+    exe = _compile(tmp_path, "abi_host_pipeline.c", cflags=("-isystem", f"{cuda}/include"),
+                   libs=(f"-L{cuda}/lib64", "-lcudart", f"-Wl,-rpath,{cuda}/lib64"))
+    r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
+    assert r.returncode == 0 and r.stdout.strip() == "ok", r.stdout + r.stderr
