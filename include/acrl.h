@@ -360,9 +360,10 @@ acrl_status acrl_reduce_loss(const float* token_loss, int64_t T, float* loss, ac
 
 /*
  * Host-buffer pipeline -- the whole on-policy pass (token statistics,
- * discrepancy, advantages, controller, gradient: the calls above) for a batch
- * whose inputs and outputs live in host memory, e.g. logits computed on or
- * offloaded to the host.  Per step the logits are uploaded in `chunks` row
+ * discrepancy, advantages, controller, gradient: the calls above, each citing
+ * its passage) for a batch whose inputs and outputs live in host memory, e.g.
+ * logits computed on or offloaded to the host.  A runtime convenience with no
+ * counterpart in the paper.  Per step the logits are uploaded in `chunks` row
  * chunks and the statistics call runs on each chunk as it lands; then the
  * discrepancy, advantage and controller calls; then the gradient call chunk
  * by chunk, each gradient chunk downloaded as soon as it is written, and the
