@@ -464,12 +464,14 @@ __global__ void lmhead_merge_kernel(const float4* __restrict__ partials, const a
     }
     LseAcc acc = lse_empty();
     float mx = -INFINITY;
+#pragma unroll 1  // tiles
     for (int n = sub; n < n_tiles; n += kMergeLanes) {
         const float4 p = partials[int64_t(n) * M + row];
         acc = lse_merge(acc, LseAcc{p.y, p.z, p.w});
         mx = fmaxf(mx, p.x);
     }
-    const unsigned group = 0xffu << (threadIdx.x & 31 & ~(kMergeLanes - 1));
+    static_assert(kMergeLanes >= 2 && kMergeLanes <= 16 && (kMergeLanes & (kMergeLanes - 1)) == 0, "lanes per row");
+    const unsigned group = ((1u << kMergeLanes) - 1u) << (threadIdx.x & 31 & ~(kMergeLanes - 1));
 #pragma unroll
     for (int m = kMergeLanes / 2; m >= 1; m >>= 1) {
         const LseAcc o{__shfl_xor_sync(group, acc.U, m), __shfl_xor_sync(group, acc.s0, m),
