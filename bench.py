@@ -46,15 +46,13 @@ FALLBACK_HBM_GBS = 6800.0
 # Kernel launches per step inside the timed region: token_stats 1, seq_discrepancy 2,
 # grpo_advantage 1, controller_step 3, loss_grad_logits 2.
 LAUNCHES_PER_STEP = 9
-# DRAM traffic of one gradient-kernel launch on the bench workload, from ncu
-# (dram__bytes_read.sum + dram__bytes_write.sum), valid only for the kernel source
-# it was taken on (sha256 of the file and the device headers, first 16 hex digits).
-# Taken with `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` (one pass) on the
-# bench workload; see profiles/dram_traffic_qwen_bench.md.
+# DRAM traffic of one launch of each kernel on its bench workload, from ncu
+# (dram__bytes_read.sum + dram__bytes_write.sum, one pass), valid only for the kernel
+# source it was taken on (sha256 of the file and the headers beside it, first 16 hex digits).
 NCU_TRAFFIC = {
     "loss_grad.cu": {"src": "fabc7049c1e852c1", "bytes_per_launch": 41.71e9 + 44.87e9},
     "token_stats.cu": {"src": "4100be30fb1483c9", "bytes_per_launch": 44.94e9 + 3.75e6},
-    # the LM-head GEMM at 32,768 x 4,096 x 151,936 (profiles/lmhead_kernel_lmhead_profile.md)
+    # the LM-head GEMM at 32,768 x 4,096 x 151,936
     "lmhead.cu": {"src": "463e708e245c83b1", "bytes_per_launch": 11.93e9 + 10.35e9},
 }
 
