@@ -116,3 +116,39 @@ def test_host_pipeline_exchange_matches_device_calls():
         assert int(bs["n_groups_valid"]) == 2 * b.Gn
     assert api.save_state(state) == api.save_state(ref.state)
     hp.close()
+
+
+def test_host_pipeline_different_batches_back_to_back():
+    """Four steps on four different batches of one shape, enqueued back to
+    back from four sets of host buffers: every upload of step k+1 lands while
+    step k still computes and downloads, so a missing order between them would
+    mix batches.  Each step must equal AcrlStep run on that step's batch."""
+    spec = W.small_variant(W.GRPO, name="hp_seq", n_prompts=3, group_size=4, len_lo=20, len_hi=150, V=8000,
+                           pad_multiple=16)
+    b = W.generate(spec, seed=47, device=DEV)
+    p = acrl.Params()
+    n = 4
+    gen = torch.Generator(device=DEV).manual_seed(5)
+    logits = [(3.0 * torch.randn((b.T, b.ld), generator=gen, device=DEV)).to(torch.bfloat16) for _ in range(n)]
+    mus = [(b.logp_mu + 0.05 * torch.randn(b.T, generator=gen, device=DEV)).clamp(max=0.0) for _ in range(n)]
+    rewards = [(torch.rand(b.S, generator=gen, device=DEV) < 0.4).float() for _ in range(n)]
+    hp = acrl.HostPipeline(b.T, b.V, b.ld, b.S, b.Gn, chunks=6)
+    state, flags = api.controller_init(p), api.new_flags()
+    small = {k: _pinned(getattr(b, k)) for k in ("ids", "mask", "seq_offsets", "group_offsets")}
+    h_logits = [_pinned(z) for z in logits]
+    h_mu = [_pinned(m) for m in mus]
+    h_r = [_pinned(r) for r in rewards]
+    grads = [torch.zeros((b.T, b.ld), dtype=torch.bfloat16, pin_memory=True) for _ in range(n)]
+    losses = [torch.zeros(1, dtype=torch.float32, pin_memory=True) for _ in range(n)]
+    for k in range(n):
+        hp.step(state, p, h_logits[k], small["ids"], small["mask"], h_mu[k], h_r[k], small["seq_offsets"],
+                small["group_offsets"], grads[k], losses[k], flags)
+    torch.cuda.synchronize()
+    ref = acrl.AcrlStep.for_batch(b, p)
+    for k in range(n):
+        ref.run(logits[k], b.ids, b.mask, mus[k], rewards[k], b.seq_offsets, b.group_offsets)
+        torch.cuda.synchronize()
+        assert torch.equal(grads[k][:, : b.V].view(torch.int16), ref.grad[:, : b.V].cpu().view(torch.int16)), k
+        assert float(losses[k][0]) == float(ref.loss[0]), k
+    assert api.save_state(state) == api.save_state(ref.state)
+    hp.close()
