@@ -21,7 +21,8 @@ readings of the CUDA path; each is listed with its reason in the design notes):
   * Sequences with no valid token are left out of Y_g and of G_g; a group with
     no valid sequence is left out of the prompt count.
   * GRPO std uses ddof=1 plus adv_eps; a group of one response gets mean 0 and
-    std 1 (so A = R) unless the ZERO rule is chosen.
+    std 1 (so A = R) unless the ZERO rule is chosen; a group whose rewards are
+    all equal gets A = 0 (decided on the rewards themselves).
   * sign(0) = 0, so A = 0 gives alpha = 0 and rho = 1.
   * min(rho, C) is evaluated as exp(min(alpha*lr, ln C)); the MIS indicator
     1{rho_i <= C} as S_i <= ln C.
@@ -34,6 +35,8 @@ readings of the CUDA path; each is listed with its reason in the design notes):
   * Any non-finite logit in a valid row makes that row's lse/logp/entropy NaN
     and sets a flag; a sampled id outside [0, V) gives logp = 0, a zero
     gradient row and a flag.
+  * A log-ratio of +inf (mu = 0 on the sampled token) follows min(rho^alpha, C)
+    with rho^0 = 1; a NaN log-ratio gets weight 0 and sets a flag.
 
 Parity status: every function here is pinned by tests that do not re-use its
 own formulas (brute force, closed forms, invariants, finite differences and
