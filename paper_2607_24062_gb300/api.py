@@ -315,6 +315,111 @@ def lmhead_merge(partials, logits, ids, mask=None, *, N=None, lse=None, logp=Non
     return lse, logp, entropy
 
 
+def lmhead_stats_noalloc(hidden, weight, ids, mask=None, *, N=None, logits=None, lse=None, logp=None, entropy=None,
+                         flags=None, stream=None):
+    """acrl_lmhead_stats_noalloc (GEMM + merge with the library's fixed scratch).
+    Returns (logits, lse, logp, entropy)."""
+    M, ldh = _rows(hidden, "hidden")
+    Nw, ldw = _rows(weight, "weight")
+    N = Nw if N is None else N
+    K = hidden.shape[1]
+    if weight.shape[1] != K:
+        raise AcrlError("hidden and weight disagree on K")
+    dev = hidden.device
+    if logits is None:
+        logits = torch.empty((M, ((N + 7) // 8) * 8), dtype=torch.bfloat16, device=dev)
+    _, ldl = _rows(logits, "logits")
+    _need(ids, torch.int32, M, "ids")
+    _opt(mask, torch.uint8, M, "mask")
+    f32 = dict(dtype=torch.float32, device=dev)
+    lse = torch.empty(M, **f32) if lse is None else _need(lse, torch.float32, M, "lse")
+    logp = torch.empty(M, **f32) if logp is None else _need(logp, torch.float32, M, "logp")
+    entropy = torch.empty(M, **f32) if entropy is None else _need(entropy, torch.float32, M, "entropy")
+    flags = _flags(flags, dev)
+    _call("acrl_lmhead_stats_noalloc", (hidden, weight, logits, ids, mask, lse, logp, entropy, flags), stream,
+          _ptr(hidden), M, K, ldh, _ptr(weight), N, ldw, _ptr(logits), ldl, _ptr(ids), _ptr(mask), _ptr(lse),
+          _ptr(logp), _ptr(entropy), _ptr(flags))
+    return logits, lse, logp, entropy
+
+
+def selftest_wait_timeout(flags, limit_ns: int, stream=None) -> None:
+    """acrl_selftest_wait_timeout: a bounded wait on a barrier nothing arrives on."""
+    _need(flags, torch.int32, 1, "flags")
+    _call("acrl_selftest_wait_timeout", (flags,), stream, _ptr(flags), int(limit_ns))
+
+
+def controller_save(state: torch.Tensor, stream=None) -> bytes:
+    """acrl_controller_save (the same as save_state)."""
+    return save_state(state, stream)
+
+
+def controller_load(blob: bytes, state: torch.Tensor | None = None, device=None, stream=None) -> torch.Tensor:
+    """acrl_controller_load (the same as load_state)."""
+    return load_state(blob, state, device, stream)
+
+
+# The host-buffer pipeline at the level of its handle (pipeline.HostPipeline wraps these).
+def host_pipeline_workspace_bytes(T: int, ld: int, S: int, Gn: int, chunks: int) -> int:
+    """acrl_host_pipeline_workspace_bytes (-1 for an invalid shape)."""
+    return int(lib().acrl_host_pipeline_workspace_bytes(T, ld, S, Gn, chunks))
+
+
+def host_pipeline_create(T: int, V: int, ld: int, S: int, Gn: int, chunks: int, workspace: torch.Tensor):
+    """acrl_host_pipeline_create on a device workspace tensor (on its device).  Returns the handle."""
+    _need(workspace, torch.uint8, max(0, host_pipeline_workspace_bytes(T, ld, S, Gn, chunks)), "workspace")
+    handle = ctypes.c_void_p()
+    with torch.cuda.device(_one_device((workspace,))):
+        check(lib().acrl_host_pipeline_create(ctypes.byref(handle), T, V, ld, S, Gn, chunks, workspace.data_ptr(),
+                                              workspace.numel()), "acrl_host_pipeline_create")
+    return handle
+
+
+def host_pipeline_step(handle, params: Params, state, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets,
+                       grad, loss, flags, stream) -> None:
+    """acrl_host_pipeline_step; host arrays as raw addresses (int), device ones as tensors."""
+    check(lib().acrl_host_pipeline_step(handle, ctypes.byref(params), _ptr(state), logits, ids, mask, logp_mu,
+                                        rewards, seq_offsets, group_offsets, grad, loss, _ptr(flags),
+                                        stream.cuda_stream), "acrl_host_pipeline_step")
+
+
+def host_pipeline_begin(handle, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets, flags,
+                        stream) -> None:
+    """acrl_host_pipeline_begin; host arrays as raw addresses (int)."""
+    check(lib().acrl_host_pipeline_begin(handle, logits, ids, mask, logp_mu, rewards, seq_offsets, group_offsets,
+                                         _ptr(flags), stream.cuda_stream), "acrl_host_pipeline_begin")
+
+
+def host_pipeline_finish(handle, params: Params, state, grad, loss, flags, stream) -> None:
+    """acrl_host_pipeline_finish; the host gradient and loss as raw addresses (int)."""
+    check(lib().acrl_host_pipeline_finish(handle, ctypes.byref(params), _ptr(state), grad, loss, _ptr(flags),
+                                          stream.cuda_stream), "acrl_host_pipeline_finish")
+
+
+def host_pipeline_batch_stats(handle) -> int:
+    """acrl_host_pipeline_batch_stats: the device address of the pipeline's batch statistics."""
+    return int(lib().acrl_host_pipeline_batch_stats(handle) or 0)
+
+
+def host_pipeline_destroy(handle) -> None:
+    """acrl_host_pipeline_destroy."""
+    check(lib().acrl_host_pipeline_destroy(handle), "acrl_host_pipeline_destroy")
+
+
+def abi_version() -> int:
+    """acrl_abi_version."""
+    return int(lib().acrl_abi_version())
+
+
+def status_string(status: int) -> str:
+    """acrl_status_string."""
+    return lib().acrl_status_string(status).decode()
+
+
+def struct_size(which: int) -> int:
+    """acrl_struct_size."""
+    return int(lib().acrl_struct_size(which))
+
+
 def read_flags(flags, stream=None) -> int:
     """acrl_read_flags (synchronises the stream)."""
     host = ctypes.c_int32(0)
@@ -338,5 +443,8 @@ def check_flags(flags, stream=None) -> None:
 
 __all__ = ["Params", "AcrlError", "token_stats", "seq_discrepancy", "grpo_advantage", "controller_init",
            "controller_step", "loss_grad_logits", "reduce_loss", "read_flags", "check_flags", "read_state", "Discrepancy",
-           "lmhead_logits_stats", "lmhead_merge", "lmhead_workspace_bytes", "save_state", "load_state",
-           "struct_buffer", "read_structs", "new_flags", "_abi"]
+           "lmhead_logits_stats", "lmhead_merge", "lmhead_workspace_bytes", "lmhead_stats_noalloc", "save_state",
+           "load_state", "controller_save", "controller_load", "selftest_wait_timeout",
+           "host_pipeline_workspace_bytes", "host_pipeline_create", "host_pipeline_step", "host_pipeline_begin",
+           "host_pipeline_finish", "host_pipeline_batch_stats", "host_pipeline_destroy", "abi_version",
+           "status_string", "struct_size", "struct_buffer", "read_structs", "new_flags", "_abi"]

@@ -21,7 +21,7 @@ from typing import Callable
 import torch
 
 from . import api
-from ._abi import BATCH_DTYPE, GRP_DTYPE, SEQ_DTYPE, STATE_DTYPE, AcrlError, Params, check
+from ._abi import BATCH_DTYPE, GRP_DTYPE, SEQ_DTYPE, STATE_DTYPE, AcrlError, Params
 
 
 class AcrlStep:
@@ -188,23 +188,19 @@ class HostPipeline:
     has been synchronised."""
 
     def __init__(self, T: int, V: int, ld: int, S: int, Gn: int, chunks: int = 16, device="cuda"):
-        L = api.lib()
-        nbytes = L.acrl_host_pipeline_workspace_bytes(T, ld, S, Gn, chunks)
+        nbytes = api.host_pipeline_workspace_bytes(T, ld, S, Gn, chunks)
         if nbytes < 0:
             raise AcrlError("acrl_host_pipeline_workspace_bytes: invalid shape")
         dev = torch.device(device)
         self.device = torch.device("cuda", torch.cuda.current_device()) if dev.index is None else dev
         self.T, self.V, self.ld, self.S, self.Gn, self.chunks = T, V, ld, S, Gn, chunks
-        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=self.device)
         self.handle = ctypes.c_void_p()
-        with torch.cuda.device(self.device):
-            check(L.acrl_host_pipeline_create(ctypes.byref(self.handle), T, V, ld, S, Gn, chunks,
-                                              self.workspace.data_ptr(), nbytes), "acrl_host_pipeline_create")
+        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=self.device)
+        self.handle = api.host_pipeline_create(T, V, ld, S, Gn, chunks, self.workspace)
 
     def batch_stats(self) -> torch.Tensor:
         """The device bytes of the pipeline's acrl_batch_stats (a view into the workspace)."""
-        addr = api.lib().acrl_host_pipeline_batch_stats(self.handle)
-        off = addr - self.workspace.data_ptr()
+        off = api.host_pipeline_batch_stats(self.handle) - self.workspace.data_ptr()
         return self.workspace[off: off + BATCH_DTYPE.itemsize]
 
     def step(self, state: torch.Tensor, params: Params, logits, ids, mask, logp_mu, rewards, seq_offsets,
@@ -230,24 +226,20 @@ class HostPipeline:
         api._need(flags, torch.int32, 1, "flags")
         if state.device != self.device or flags.device != self.device:
             raise AcrlError("state / flags: expected on the pipeline's device")
-        L = api.lib()
         with torch.cuda.device(self.device):
             s = torch.cuda.current_stream(self.device) if stream is None else stream
             if exchange is None:
-                check(L.acrl_host_pipeline_step(self.handle, ctypes.byref(params), state.data_ptr(), *ptrs,
-                                                flags.data_ptr(), s.cuda_stream), "acrl_host_pipeline_step")
+                api.host_pipeline_step(self.handle, params, state, *ptrs, flags, s)
                 return
-            check(L.acrl_host_pipeline_begin(self.handle, *ptrs[:7], flags.data_ptr(), s.cuda_stream),
-                  "acrl_host_pipeline_begin")
+            api.host_pipeline_begin(self.handle, *ptrs[:7], flags, s)
             with torch.cuda.stream(s):
                 exchange(self.batch_stats())
-            check(L.acrl_host_pipeline_finish(self.handle, ctypes.byref(params), state.data_ptr(), ptrs[7], ptrs[8],
-                                              flags.data_ptr(), s.cuda_stream), "acrl_host_pipeline_finish")
+            api.host_pipeline_finish(self.handle, params, state, ptrs[7], ptrs[8], flags, s)
 
     def close(self) -> None:
-        if self.handle:
+        if getattr(self, "handle", None):
             h, self.handle = self.handle, ctypes.c_void_p()
-            check(api.lib().acrl_host_pipeline_destroy(h), "acrl_host_pipeline_destroy")
+            api.host_pipeline_destroy(h)
 
     def __del__(self):
         try:

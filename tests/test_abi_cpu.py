@@ -28,6 +28,13 @@ def test_exports_every_declared_function(L):
     assert set(declared) == set(_abi.SIGNATURES)
 
 
+def test_binding_has_a_function_per_entry_point():
+    """The binding mirrors the header: acrl_x is api.x, for every declaration."""
+    from paper_2607_24062_gb300 import api
+    missing = [n for n in _abi.header_functions() if not callable(getattr(api, n[len("acrl_"):], None))]
+    assert not missing, missing
+
+
 def test_abi_version_and_layouts(L):
     assert L.acrl_abi_version() == 2
     assert L.acrl_struct_size(0) == ctypes.sizeof(_abi.Params) == 64

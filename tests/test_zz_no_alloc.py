@@ -71,3 +71,13 @@ def test_noalloc_refuses_oversized_problem():
                                               H.data_ptr(), H.data_ptr(), api.new_flags().data_ptr(), None)
     assert st == _abi.ERR_SCRATCH_TOO_SMALL
     assert b"scratch" in _abi.lib().acrl_status_string(st)
+
+
+def test_noalloc_through_the_binding():
+    H, Wt, ids, mask = _problem(300, 2000, 72, 5)
+    logits, lse, logp, ent = api.lmhead_stats_noalloc(H, Wt, ids, mask, N=2000)
+    logits2, lse2, logp2, ent2, _ = _noalloc(H, Wt, 2000, ids, mask)
+    torch.cuda.synchronize()
+    assert torch.equal(logits[:, :2000], logits2[:, :2000])
+    for a, b in ((lse, lse2), (logp, logp2), (ent, ent2)):
+        assert torch.equal(a, b)
