@@ -677,3 +677,38 @@ def test_importance_weights_from_log_probs(mode):
         coef = O.loss_coefficients(w, adv, mask, so, seq, grp, batch, op)
         assert_close_rel(host(r.coef), coef, floor=1e-12, what="coef")
         assert_close_rel(api.read_state(state)["X"], ostate.X, floor=1e-12, what="X")
+
+
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 16383, 16384, 16385, 65535, 65536, 65537, 65544])
+def test_row_size_class_boundaries(V):
+    """Vocabularies at the edges of the row-team size classes (one warp up to
+    16,384 columns, 64 threads up to 65,536, 128 above for the statistics;
+    one warp, then 512 threads for the gradient) and of the 8-column vectors:
+    statistics and gradient against the oracle on every element, with the
+    lse recomputed in the gradient kernel as well."""
+    T = 37
+    ld = ((V + 7) // 8) * 8
+    gen = torch.Generator(device=DEV).manual_seed(V)
+    logits = (2.0 * torch.randn((T, ld), generator=gen, device=DEV)).to(torch.bfloat16)
+    ids = torch.randint(0, V, (T,), generator=gen, device=DEV, dtype=torch.int32)
+    mask = (torch.rand(T, generator=gen, device=DEV) < 0.85).to(torch.uint8)
+    coef = torch.randn(T, generator=gen, device=DEV) * mask.float()
+    flags = api.new_flags()
+    lse, logp, H = api.token_stats(logits, ids, mask, V=V, flags=flags)
+    z = rows_f64(logits, np.arange(T), V)
+    olse, ologp, oH, _ = O.token_stats(z, host(ids), host(mask))
+    assert_close_abs(host(lse), olse, TOL_LOGP, "lse")
+    assert_close_abs(host(logp), ologp, TOL_LOGP, "logp")
+    assert_close_rel(host(H), oH, floor=1e-5, what="entropy")
+    m = host(mask).astype(bool)
+    p = np.exp(z - olse[:, None])
+    onehot = np.zeros((T, V))
+    onehot[np.arange(T), host(ids)] = 1.0
+    want = host(coef).astype(np.float64)[:, None] * (p - onehot)
+    want[~m] = 0.0
+    for recompute in (False, True):
+        grad, _, _ = api.loss_grad_logits(logits, ids, mask, None if recompute else lse, None, coef, 0.2, V=V,
+                                          flags=flags)
+        assert_grad_rows(grad_rows(grad, np.arange(T), V), want, host(coef), host(ids), what=f"grad (recompute "
+                         f"{recompute})")
+    assert api.read_flags(flags) == 0
