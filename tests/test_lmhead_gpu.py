@@ -41,9 +41,11 @@ def _check_logits(got_bf16, ref, abs_sum, K, what="logits"):
 
 # also: one row and a vocabulary narrower than a 32-column store block; an odd number of row tiles (the second
 # CTA of the last cluster has no rows) with a ragged K; K narrower than one 64-column slab; 66 row tiles, i.e.
-# three bands of row-tile pairs (16, 16 and a ragged 1) with a ragged last tile
+# three bands of row-tile pairs (16, 16 and a ragged 1) with a ragged last tile; one short of / one past the
+# 128-row and 256-column tile edges with K off the 64-column slab
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (200, 1000, 328), (384, 2304, 4096), (130, 151936, 64),
-                                   (1, 8, 64), (257, 520, 72), (5, 40, 8), (8322, 1000, 64)])
+                                   (1, 8, 64), (257, 520, 72), (5, 40, 8), (8322, 1000, 64),
+                                   (127, 255, 16), (129, 257, 136), (256, 512, 200), (255, 33, 24)])
 def test_lmhead_small_shapes(M, N, K):
     gen = torch.Generator(device=DEV).manual_seed(M * 7 + N + K)
     H = torch.randn((M, K), generator=gen, device=DEV).to(torch.bfloat16)
@@ -62,10 +64,16 @@ def test_lmhead_small_shapes(M, N, K):
     assert_close_abs(host(lse), olse, 1e-5 + 1e-6 * np.abs(olse), "lse (stored logits)")
     assert_close_abs(host(logp), ologp, 2e-5, "logp (stored logits)")
     assert_close_rel(host(ent), oH, rel=1e-4, floor=1e-6, what="entropy (stored logits)")
-    # ... and against the oracle's own chain
+    # ... and against the oracle's own chain.  A logit whose exact value sits within the fp32 accumulation error
+    # of a bf16 rounding boundary may be stored one ulp off the oracle's rounding (both roundings are valid,
+    # _check_logits allows it); lse moves by sum_j p_j |dz_j| and log p by that plus |dz_a| in such a row.
     olse, ologp, oH, _ = O.token_stats(z, host(ids), host(mask))
-    assert_close_abs(host(lse), olse, TOL_LOGP, "lse")
-    assert_close_abs(host(logp), ologp, TOL_LOGP, "logp")
+    dz = np.abs(zg - z)
+    p = np.exp(z - olse[:, None])
+    shift = (p * dz).sum(axis=1)
+    a = host(ids)
+    assert_close_abs(host(lse), olse, TOL_LOGP + shift, "lse")
+    assert_close_abs(host(logp), ologp, TOL_LOGP + shift + dz[np.arange(M), a], "logp")
     assert_close_rel(host(ent), oH, floor=1e-5, what="entropy")
 
 
@@ -126,12 +134,17 @@ def test_lmhead_workload_full_chain():
     del Wf
     _check_logits(logits[torch.as_tensor(rows, device=DEV), :b.N], z, abs_sum, b.K, "logits (sampled rows)")
     olse, ologp, oH, _ = O.token_stats(z, host(b.ids)[rows], mask[rows])
-    assert_close_abs(host(lse)[rows], olse, TOL_LOGP, "lse")
-    assert_close_abs(host(logp)[rows], ologp, TOL_LOGP, "logp")
+    # a stored logit one bf16 ulp off the oracle's rounding (both valid) moves lse by p_j |dz_j| and log p by
+    # that plus |dz_a|: the statistics may differ from the oracle's chain by that much beyond TOL_LOGP
+    zg = rows_f64(logits, rows, b.N)
+    dz = np.abs(zg - z)
+    shift = (np.exp(z - olse[:, None]) * dz).sum(axis=1)
+    a = host(b.ids)[rows]
+    assert_close_abs(host(lse)[rows], olse, TOL_LOGP + shift, "lse")
+    assert_close_abs(host(logp)[rows], ologp, TOL_LOGP + shift + dz[np.arange(len(rows)), a], "logp")
     assert_close_rel(host(ent)[rows], oH, floor=1e-5, what="entropy")
     # The gradient pass is judged on the logits it consumed: a logit one bf16 ulp
     # away (about 0.1 % of them, see _check_logits) moves its p by e^ulp, ~1-2 %.
-    zg = rows_f64(logits, rows, b.N)
     glse, _, _, _ = O.token_stats(zg, host(b.ids)[rows], mask[rows])
     lse_full = np.zeros(b.T)
     lse_full[rows] = glse
