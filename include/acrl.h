@@ -11,7 +11,9 @@
  *
  * Conventions shared by every call:
  *   - Pointers documented "device" must be device memory of the current CUDA
- *     device (or managed memory).  The caller owns every buffer; the library
+ *     device (managed memory is accepted too, except by the LM-head calls,
+ *     whose tensor-core copies need plain device memory of the current
+ *     device: they check this on the host).  The caller owns every buffer; the library
  *     allocates no device memory and keeps no global state, except the fixed
  *     scratch array of acrl_lmhead_stats_noalloc (documented there).  The
  *     host-buffer pipeline's handle owns two streams and its events, made by
@@ -336,7 +338,11 @@ acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params
  *           NULL to recompute it here (the cached-old path: a second sweep
  *           over each row).
  *   old_logp  device float [T] log pi_old(a_t), or NULL for r = 1.
- *   coef    device float [T] from acrl_controller_step.
+ *   coef    device float [T]: acrl_controller_step's `coef` output for the
+ *           same batch (the same rows, in the same order).  It carries
+ *           m_t w_t A_i / norm_t, and its sign is the sign of A_i, which the
+ *           clip gate g_t reads (A_i >= 0: r <= 1+eps; A_i < 0: r >= 1-eps);
+ *           coef_t = 0 carries no policy gradient, whatever A_i was.
  *   entropy, ent_coef  device float [T] (acrl_token_stats' entropy and
  *           acrl_controller_step's ent_coef), both NULL for no entropy bonus.
  *   clip_eps  the eps of Eq. grpo_objective.
@@ -440,6 +446,11 @@ acrl_status acrl_host_pipeline_destroy(acrl_host_pipeline* pipeline);
  *   logits   device bf16 [M, ldl] output (ldl >= N, multiple of 8).
  *   partials device float4 workspace of acrl_lmhead_workspace_bytes(M, N)
  *            bytes, layout [ceil(N/256)][M]; owned by the caller.
+ * hidden, weight and logits must be device memory of the current device:
+ * managed memory, host memory (page-locked or not) and another GPU's memory
+ * are refused with ACRL_ERR_INVALID_ARG (checked with cudaPointerGetAttributes
+ * before anything is launched), since the tensor-core copies are encoded over
+ * these pointers.
  * Pipeline waits are time-bounded: ACRL_FLAG_TIMEOUT means the outputs of this
  * call are invalid.  Requires an sm_100-family GPU (built for sm_103a).
  */
@@ -474,11 +485,16 @@ acrl_status acrl_lmhead_merge(const float* partials, const acrl_bf16* logits, in
  *   N = 151,936 or M <= 8388 at N = 32,000; larger problems return
  *   ACRL_ERR_SCRATCH_TOO_SMALL before anything is launched.
  *   The first call on each device looks up the array's device address with
- *   that device current; make that first call before any stream capture.
+ *   that device current and keeps it for the life of the process; make that
+ *   first call before any stream capture.  A device reset (cudaDeviceReset,
+ *   or the primary context torn down and made again) invalidates the kept
+ *   address: do not call this entry point on a device after resetting it.
  *   All calls share the array: calls that overlap on the GPU (different
  *   streams, or different host threads, on the same device) race on it and
  *   must be ordered by the caller.  Nothing in it needs clearing between calls.
- *   Arguments, outputs and flags are those of the two calls it combines.
+ *   Arguments, outputs and flags are those of the two calls it combines,
+ *   including the rule that hidden, weight and logits be device memory of
+ *   the current device.
  */
 #define ACRL_LMHEAD_NOALLOC_SCRATCH_BYTES (16LL << 20)
 acrl_status acrl_lmhead_stats_noalloc(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t ldh,

@@ -5,29 +5,28 @@
 // lse, the sampled token's log-prob and the entropy without reading the logits
 // again.
 //
-// Blackwell path: a persistent kernel in clusters of two CTAs, one CTA per SM,
-// warp-specialised.  The two CTAs of a cluster work on the two row tiles of a
-// pair that share one weight tile.
+// Blackwell path: a persistent kernel, one CTA per SM, warp-specialised.
 //   warp 0     one thread issues TMA tile loads (128B-swizzled) into a 4-stage
-//              shared-memory ring of A 128x64 + B 256x64 bf16: its own A, and
-//              its half of B multicast into both CTAs of the cluster;
+//              shared-memory ring of A 128x64 + B 256x64 bf16;
 //   warp 1     one thread issues tcgen05.mma (M=128, N=256, K=16, kind::f16)
 //              into a TMEM accumulator and commits each stage back to the
-//              producers of both CTAs; two 256-column accumulators alternate
-//              between tiles;
+//              producer; two 256-column accumulators alternate between tiles;
 //   warps 2-5  the epilogue: tcgen05.ld of the accumulator (each thread one
 //              row), round to bf16, fold the statistics, and write the logits
 //              through shared memory with TMA bulk tensor stores (32 x 32
 //              blocks, two staging buffers per warp).
 // Tiles are visited in bands of 32 row tiles so that the weight tiles in
-// flight are shared through L2 by the clusters working on the same band.
+// flight are shared through L2 by the CTAs working on the same band.  Every
+// CTA loads its operands from this GPU's memory into its own shared memory
+// only (the tensor maps are encoded over pointers that the entry points have
+// checked to be device memory of the current device).
 // Every wait on an mbarrier is bounded in time; on expiry the kernel raises
 // ACRL_FLAG_TIMEOUT, lets the copies it issued land, and exits after freeing
-// its TMEM.  The two CTAs meet at a cluster barrier after initialising their
-// barriers and again before either frees its TMEM or exits, so neither writes
-// into a peer that has gone.
+// its TMEM.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+
+#include <initializer_list>
 
 #include "acrl_device.cuh"
 #include "acrl_host.h"
@@ -164,8 +163,7 @@ __device__ __forceinline__ void bulk_wait_read() {
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // ---------------------------------------------------------------------------
-// tile schedule: bands of BAND row tiles (row-tile pairs for the clusters),
-// all column tiles of a band in turn
+// tile schedule: bands of BAND row tiles, all column tiles of a band in turn
 // ---------------------------------------------------------------------------
 
 template <int BAND = kBandM>
@@ -176,39 +174,6 @@ __device__ __forceinline__ void tile_coords(int t, int m_tiles, int n_tiles, int
     const int bm = min(BAND, m_tiles - band * BAND);
     m = band * BAND + r % bm;
     n = r / bm;
-}
-
-// ---------------------------------------------------------------------------
-// the cluster of two
-// ---------------------------------------------------------------------------
-
-__device__ __forceinline__ uint32_t cluster_rank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-
-__device__ __forceinline__ void cluster_sync() {
-    asm volatile("barrier.cluster.arrive.release;\nbarrier.cluster.wait.acquire;" ::: "memory");
-}
-
-// Tile load written at the same shared-memory offset in every CTA of `mask`,
-// each CTA's barrier at `bar`'s offset counting the bytes it received.
-__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
-                                               uint16_t mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, {%2, "
-        "%3}], [%4], %5;" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "h"(mask)
-        : "memory");
-}
-// Arrive on `bar` in both CTAs once this thread's MMAs so far have completed.
-__device__ __forceinline__ void mma_commit_mc(uint64_t* bar) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-            smem_u32(bar)),
-        "h"(uint16_t(3))
-        : "memory");
 }
 
 __device__ __forceinline__ void give_up(volatile int32_t* abort, int32_t* flags) {
@@ -229,12 +194,9 @@ __device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t
     uint32_t phase = 0;
     long issued = 0;
     bool ok = true;
-    const uint32_t rank = cluster_rank();
-    const int m_pairs = (m_tiles + 1) / 2;
-    for (int t = int(blockIdx.x >> 1); t < total && ok; t += int(gridDim.x >> 1)) {
-        int mp, n;
-        tile_coords<kBandM / 2>(t, m_pairs, n_tiles, mp, n);
-        const int m = 2 * mp + int(rank);
+    for (int t = int(blockIdx.x); t < total && ok; t += int(gridDim.x)) {
+        int m, n;
+        tile_coords(t, m_tiles, n_tiles, m, n);
         for (int kk = 0; kk < k_iters; ++kk) {
             if (!mbar_try_wait(&bars->empty[stage], phase ^ 1u) &&
                 !wait_phase(&bars->empty[stage], phase ^ 1u, abort)) {
@@ -244,8 +206,7 @@ __device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t
             }
             mbar_expect_tx(&bars->full[stage], R::kStageBytes);
             tma_load_2d(sA + stage * R::kABytes, tmA, &bars->full[stage], kk * R::kBK, m * kBM);
-            tma_load_2d_mc(sB + stage * R::kBBytes + int(rank) * (R::kBBytes / 2), tmB, &bars->full[stage], kk * R::kBK,
-                           n * kBN + int(rank) * (kBN / 2), uint16_t(3));
+            tma_load_2d(sB + stage * R::kBBytes, tmB, &bars->full[stage], kk * R::kBK, n * kBN);
             ++issued;
             if (++stage == kStages) {
                 stage = 0;
@@ -272,7 +233,7 @@ __device__ void mma_issuer(uint8_t* sA, uint8_t* sB, typename R::Barriers* bars,
     int acc = 0;
     uint32_t acc_phase = 0;
     bool ok = true;
-    for (int t = int(blockIdx.x >> 1); t < total && ok; t += int(gridDim.x >> 1)) {
+    for (int t = int(blockIdx.x); t < total && ok; t += int(gridDim.x)) {
         if (!wait_phase(&bars->tempty[acc], acc_phase ^ 1u, abort)) {
             give_up(abort, flags);
             break;
@@ -292,7 +253,7 @@ __device__ void mma_issuer(uint8_t* sA, uint8_t* sB, typename R::Barriers* bars,
 #pragma unroll
             for (int k16 = 0; k16 < R::kBK / 16; ++k16)  // 16 columns = 32 bytes = 2 descriptor units
                 mma_bf16(d, ad + uint64_t(2 * k16), bd + uint64_t(2 * k16), (kk | k16) != 0);
-            mma_commit_mc(&bars->empty[stage]);
+            mma_commit(&bars->empty[stage]);
             if (++stage == kStages) {
                 stage = 0;
                 phase ^= 1u;
@@ -322,12 +283,9 @@ __device__ void epilogue(Bars* bars, uint32_t tmem, const CUtensorMap* tmC, uint
     int buf = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
-    const uint32_t rank = cluster_rank();
-    const int m_pairs = (m_tiles + 1) / 2;
-    for (int t = int(blockIdx.x >> 1); t < total; t += int(gridDim.x >> 1)) {
-        int mp, n;
-        tile_coords<kBandM / 2>(t, m_pairs, n_tiles, mp, n);
-        const int m = 2 * mp + int(rank);
+    for (int t = int(blockIdx.x); t < total; t += int(gridDim.x)) {
+        int m, n;
+        tile_coords(t, m_tiles, n_tiles, m, n);
         const bool ready = wait_phase(&bars->tfull[acc], acc_phase, abort);
         if (!__all_sync(0xffffffffu, ready)) {
             give_up(abort, flags);
@@ -385,7 +343,7 @@ __device__ void epilogue(Bars* bars, uint32_t tmem, const CUtensorMap* tmC, uint
 }
 
 template <class R>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     lmhead_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                   const __grid_constant__ CUtensorMap tmC, int M, int N, int K, float4* __restrict__ partials,
                   int32_t* flags) {
@@ -399,13 +357,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     Barriers* bars = reinterpret_cast<Barriers*>(sOut + kOutBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m_tiles = (M + kBM - 1) / kBM, n_tiles = (N + kBN - 1) / kBN;
-    const int total = ((m_tiles + 1) / 2) * n_tiles;  // tile pairs sharing a weight tile
+    const int total = m_tiles * n_tiles;
     const int k_iters = (K + R::kBK - 1) / R::kBK;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&bars->full[s], 1);
-            mbar_init(&bars->empty[s], 2);  // released by both CTAs' MMAs
+            mbar_init(&bars->empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&bars->tfull[b], 1);
@@ -413,7 +371,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         mbar_init(&bars->mma_done, 1);
         bars->abort = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");  // visible to the async proxy
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmC)) : "memory");
@@ -426,7 +384,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
     tc_fence_before();
     __syncthreads();
-    cluster_sync();
     tc_fence_after();
     const uint32_t tmem = bars->tmem_base;
 
@@ -439,7 +396,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
     tc_fence_before();
     __syncthreads();
-    cluster_sync();
     if (warp == 2) {
         tc_fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
@@ -508,35 +464,56 @@ bool encode_map(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Tensor maps, shared-memory opt-in and the persistent launch (clusters of two
-// CTAs, one CTA per SM, fewer if there are fewer tile pairs).  Arguments are
-// checked by the callers.
+// Tensor maps, shared-memory opt-in and the persistent launch (one CTA per SM,
+// fewer if there are fewer tiles).  Arguments, including where the operands
+// live, are checked by the callers.
 template <class R>
 acrl_status launch_lmhead(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t ldh, const acrl_bf16* weight,
                           int64_t N, int64_t ldw, acrl_bf16* logits, int64_t ldl, float4* partials, int32_t* flags,
                           cudaStream_t s) {
     CUtensorMap tmA, tmB, tmC;
     if (!encode_map(&tmA, hidden, uint64_t(M), uint64_t(K), uint64_t(ldh), kBM, R::kBK, R::kTmaSwizzle) ||
-        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN / 2, R::kBK, R::kTmaSwizzle) ||
+        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN, R::kBK, R::kTmaSwizzle) ||
         !encode_map(&tmC, logits, uint64_t(M), uint64_t(N), uint64_t(ldl), 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
         return ACRL_ERR_CUDA;
     if (cudaFuncSetAttribute(lmhead_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, R::kSmemBytes) !=
         cudaSuccess)
         return ACRL_ERR_CUDA;
-    // pairs of row tiles x column tiles; as many clusters as can be resident at once
-    const int64_t total = (((M + kBM - 1) / kBM + 1) / 2) * ((N + kBN - 1) / kBN);
-    if (total > kMaxGrid / 2) return ACRL_ERR_INVALID_ARG;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(2 * 1024, 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = R::kSmemBytes;
-    cfg.stream = s;
-    int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, lmhead_kernel<R>, &cfg) != cudaSuccess || clusters < 1)
+    const int64_t total = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
+    if (total > kMaxGrid) return ACRL_ERR_INVALID_ARG;
+    int dev = 0, sms = 0, per_sm = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lmhead_kernel<R>, kThreads, R::kSmemBytes) !=
+            cudaSuccess ||
+        per_sm < 1)
         return ACRL_ERR_CUDA;
-    const int grid = int(2 * (total < clusters ? total : clusters));
+    const int64_t resident = int64_t(sms) * per_sm;
+    const int grid = int(total < resident ? total : resident);
     lmhead_kernel<R><<<grid, kThreads, R::kSmemBytes, s>>>(tmA, tmB, tmC, int(M), int(N), int(K), partials, flags);
     return launch_status();
+}
+
+// True when every pointer is device memory of the current device: not managed
+// memory, not host memory and not a peer GPU's memory.  The GEMM's tensor maps
+// are encoded over these pointers, and its TMA copies must stay within this
+// GPU's own memory.  A failed query counts as "no" and leaves no error behind
+// for a later launch check.
+bool operands_on_current_device(std::initializer_list<const void*> ptrs) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return false;
+    }
+    for (const void* p : ptrs) {
+        cudaPointerAttributes a{};
+        if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+            (void)cudaGetLastError();
+            return false;
+        }
+        if (a.type != cudaMemoryTypeDevice || a.device != dev) return false;
+    }
+    return true;
 }
 
 }  // namespace
@@ -560,6 +537,7 @@ extern "C" acrl_status acrl_lmhead_logits_stats(const acrl_bf16* hidden, int64_t
     if (!hidden || !weight || !logits || !partials) return ACRL_ERR_INVALID_ARG;
     if (!aligned16(hidden) || !aligned16(weight) || !aligned16(logits) || !aligned16(partials))
         return ACRL_ERR_INVALID_ARG;
+    if (!operands_on_current_device({hidden, weight, logits})) return ACRL_ERR_INVALID_ARG;
     return launch_lmhead<LmRing>(hidden, M, K, ldh, weight, N, ldw, logits, ldl, reinterpret_cast<float4*>(partials),
                                  dev_flags, reinterpret_cast<cudaStream_t>(stream));
 }
@@ -626,6 +604,7 @@ extern "C" acrl_status acrl_lmhead_stats_noalloc(const acrl_bf16* hidden, int64_
     if (M == 0) return ACRL_OK;
     if (!hidden || !weight || !logits || !ids || !lse || !logp || !entropy) return ACRL_ERR_INVALID_ARG;
     if (!aligned16(hidden) || !aligned16(weight) || !aligned16(logits)) return ACRL_ERR_INVALID_ARG;
+    if (!operands_on_current_device({hidden, weight, logits})) return ACRL_ERR_INVALID_ARG;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return ACRL_ERR_CUDA;
     float4* partials = noalloc_scratch(dev);

@@ -10,6 +10,10 @@ if ROOT not in sys.path:
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built library")
+    # name every skipped test (or module) and its reason in the summary
+    chars = getattr(config.option, "reportchars", "") or ""
+    if not any(c in chars for c in "sSaA"):
+        config.option.reportchars = chars + "s"
 
 
 def pytest_collection_modifyitems(config, items):

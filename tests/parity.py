@@ -16,8 +16,12 @@ Integer outputs (counts, group indices, flags) must match exactly."""
 
 from __future__ import annotations
 
+import atexit
+import concurrent.futures
+import multiprocessing
+import os
+
 import numpy as np
-import torch
 
 import oracle as O
 
@@ -38,14 +42,20 @@ def oracle_params(p) -> O.Params:
                     singleton_rule=int(p.singleton_rule), calib_steps=int(p.calib_steps), X_init=float(p.X_init))
 
 
-def rows_f64(logits: torch.Tensor, rows, V: int) -> np.ndarray:
+def rows_bits(t, rows, V: int) -> np.ndarray:
+    """The raw bf16 bits (uint16) of `rows` of a [T, ld] tensor, first V columns."""
+    import torch
+    idx = torch.as_tensor(np.asarray(rows, dtype=np.int64), device=t.device)
+    return t.index_select(0, idx)[:, :V].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def rows_f64(logits, rows, V: int) -> np.ndarray:
     """Exact float64 copy of the bf16 logits of `rows` (first V columns)."""
-    idx = torch.as_tensor(np.asarray(rows, dtype=np.int64), device=logits.device)
-    bits = logits.index_select(0, idx)[:, :V].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
-    return O.bf16_bits_to_f64(bits)
+    return O.bf16_bits_to_f64(rows_bits(logits, rows, V))
 
 
-def grad_rows(grad: torch.Tensor, rows, V: int) -> np.ndarray:
+def grad_rows(grad, rows, V: int) -> np.ndarray:
+    import torch
     idx = torch.as_tensor(np.asarray(rows, dtype=np.int64), device=grad.device)
     return grad.index_select(0, idx)[:, :V].float().cpu().numpy().astype(np.float64)
 
@@ -127,3 +137,103 @@ def assert_loss(got, ref, ref_token_loss, what="loss"):
     batches whose token losses cancel (e.g. every weight 1: sum_i A_i = 0)."""
     floor = 1e-6 * float(np.nansum(np.abs(np.asarray(ref_token_loss, dtype=np.float64)))) + 1e-30
     assert_close_rel(got, ref, floor=floor, what=what)
+
+
+# --------------------------------------------------------------------------
+# the vocabulary-wide outputs of many rows, checked in parallel
+# --------------------------------------------------------------------------
+
+_POOL = None
+
+
+def oracle_pool():
+    """Worker processes for the oracle's per-row work, one per host core (at
+    most 16).  Spawned, so that none inherits this process's CUDA context;
+    they import numpy and the oracle only."""
+    global _POOL
+    if _POOL is None:
+        n = max(1, min(16, len(os.sched_getaffinity(0))))
+        _POOL = (concurrent.futures.ProcessPoolExecutor(max_workers=n,
+                                                        mp_context=multiprocessing.get_context("spawn")), n)
+        atexit.register(_POOL[0].shutdown)
+    return _POOL
+
+
+def _vocab_rows_block(zbits, gbits, rr, T, ids_r, mask_r, w_r, coef_r, adv, so, seq, grp, batch, op, lse_g, logp_g,
+                      ent_g):
+    """One block of rows in a worker: the oracle's log-softmax of the exact
+    float64 logits against the GPU's lse / logp / entropy, then the oracle's
+    gradient rows (Eq. ACRL) against the GPU's bf16 gradient rows.  Returns
+    (rows, oracle logp, oracle entropy)."""
+    z = O.bf16_bits_to_f64(zbits)
+    olse, ologp, oH, f = O.token_stats(z, ids_r, mask_r)
+    assert f == 0, f"oracle flags {f}"
+    assert_close_abs(lse_g, olse, TOL_LOGP, "lse")
+    assert_close_abs(logp_g, ologp, TOL_LOGP, "logp")
+    assert_close_rel(ent_g, oH, floor=1e-5, what="entropy")
+    if gbits is not None:
+        full = np.zeros(T)
+        full[rr] = olse
+        ids_full = np.zeros(T, dtype=np.int64)
+        ids_full[rr] = ids_r
+        mask_full = np.zeros(T, dtype=np.uint8)
+        mask_full[rr] = mask_r
+        w_full = np.zeros(T)
+        w_full[rr] = w_r
+        ograd, _, _ = O.loss_grad_logits(z, ids_full, mask_full, full, None, adv, w_full, so, seq, grp, batch, op,
+                                         rows=rr)
+        assert_grad_rows(O.bf16_bits_to_f64(gbits), ograd, coef_r, ids_r)
+    return rr, ologp, oH
+
+
+class VocabRowCheck:
+    """Element-by-element check of the vocabulary-wide outputs (a1: lse, logp,
+    entropy; a6: the gradient rows) of sampled rows against the oracle's own
+    float64 log-softmax and gradient, in blocks of rows spread over the
+    oracle pool.  `ref` holds the O(T) references the gradient needs (adv, w,
+    coef, seq, grp, batch).  The oracle's logp and entropy of every checked
+    row are kept (`oracle_logp`, `oracle_entropy`) for the oracle's own chain
+    on whole responses."""
+
+    def __init__(self, T, ids, mask, seq_offsets, ref, op, block=256):
+        self.pool, self.n = oracle_pool()
+        self.T, self.ids, self.mask = T, np.asarray(ids), np.asarray(mask)
+        self.so = np.asarray(seq_offsets)
+        self.ref, self.op, self.block = ref, op, block
+        self.pending = set()
+        self.oracle_logp, self.oracle_entropy = {}, {}
+        self.rows_checked = 0
+
+    def _collect(self, futures):
+        for f in futures:
+            rr, lp, H = f.result()      # re-raises a worker's AssertionError here
+            self.oracle_logp.update(zip(rr.tolist(), lp.tolist()))
+            self.oracle_entropy.update(zip(rr.tolist(), H.tolist()))
+            self.rows_checked += len(rr)
+
+    def submit(self, logits, V, rows, lse, logp, entropy, grad=None, grad_row0=0):
+        """Queue `rows` (global row indices) for checking.  `grad` holds the
+        gradient rows from global row `grad_row0` on (a chunk buffer), or is
+        None to check the statistics alone.  The rows' data are copied to the
+        host before this returns, so the buffers may be reused."""
+        rows = np.asarray(rows, dtype=np.int64)
+        lse_h, logp_h, ent_h = host(lse), host(logp), host(entropy)
+        r = self.ref
+        for k in range(0, len(rows), self.block):
+            rr = rows[k:k + self.block]
+            zb = rows_bits(logits, rr, V)
+            gb = None if grad is None else rows_bits(grad, rr - grad_row0, V)
+            while len(self.pending) >= 2 * self.n:
+                done, self.pending = concurrent.futures.wait(self.pending,
+                                                             return_when=concurrent.futures.FIRST_COMPLETED)
+                self._collect(done)
+            self.pending.add(self.pool.submit(
+                _vocab_rows_block, zb, gb, rr, self.T, self.ids[rr], self.mask[rr], r["w"][rr], r["coef"][rr],
+                r["adv"], self.so, r["seq"], r["grp"], r["batch"], self.op, lse_h[rr], logp_h[rr], ent_h[rr]))
+
+    def finish(self):
+        """Wait for every queued block; returns the number of rows checked."""
+        done, _ = concurrent.futures.wait(self.pending)
+        self.pending = set()
+        self._collect(done)
+        return self.rows_checked

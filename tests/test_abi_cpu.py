@@ -103,6 +103,12 @@ def test_host_side_rejections(L):
     assert L.acrl_reduce_loss(None, 4, fake, None) == E
     assert L.acrl_selftest_wait_timeout(None, 1000, None) == E
     assert L.acrl_selftest_wait_timeout(fake, 3_000_000_000, None) == E
+    # the LM-head calls encode their tensor-core copies over hidden, weight and logits, which must be device memory
+    # of the current device: pointers that cannot be shown to be (here: no device, or a host address) are refused
+    # before anything is launched
+    assert L.acrl_lmhead_logits_stats(fake, 4, 64, 64, fake, 256, 64, fake, 256, fake, fake, None) == E
+    assert L.acrl_lmhead_stats_noalloc(fake, 4, 64, 64, fake, 256, 64, fake, 256, fake, None, fake, fake, fake, fake,
+                                       None) == E
 
 
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):

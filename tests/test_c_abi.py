@@ -14,11 +14,21 @@ CDIR = os.path.join(ROOT, "tests", "c")
 LIBDIR = os.path.dirname(build.LIB)
 
 
+def _missing(what):
+    """A C client that cannot be built: a failure where a GPU is present (the
+    C clients are the evidence that the boundary works from plain C), a
+    skip on a CPU-only machine."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.fail(f"{what}: the C99 clients must build and run on a GPU machine")
+    pytest.skip(what)
+
+
 def _compile(tmp_path, src, cflags=(), libs=()):
     if shutil.which("gcc") is None:
-        pytest.skip("gcc not available")
+        _missing("gcc not available")
     if shutil.which("nvcc") is None and not build.up_to_date():
-        pytest.skip("no nvcc to build the library")
+        _missing("no nvcc to build the library")
     build.build()
     exe = str(tmp_path / os.path.splitext(src)[0])
     cmd = ["gcc", "-std=c99", "-Wall", "-Wextra", "-Werror", "-pedantic", f"-I{ROOT}/include", *cflags,

@@ -16,7 +16,7 @@ from parity import (TOL_LOGP, assert_close_abs, assert_close_rel, assert_grad_ro
 pytestmark = pytest.mark.gpu
 
 import paper_2607_24062_gb300 as acrl  # noqa: E402
-from paper_2607_24062_gb300 import api  # noqa: E402
+from paper_2607_24062_gb300 import _abi, api  # noqa: E402
 
 DEV = "cuda"
 
@@ -39,10 +39,10 @@ def _check_logits(got_bf16, ref, abs_sum, K, what="logits"):
     assert np.mean(got == ref) > 0.99
 
 
-# also: one row and a vocabulary narrower than a 32-column store block; an odd number of row tiles (the second
-# CTA of the last cluster has no rows) with a ragged K; K narrower than one 64-column slab; 66 row tiles, i.e.
-# three bands of row-tile pairs (16, 16 and a ragged 1) with a ragged last tile; one short of / one past the
-# 128-row and 256-column tile edges with K off the 64-column slab
+# also: one row and a vocabulary narrower than a 32-column store block; an odd number of row tiles with a
+# ragged K; K narrower than one 64-column slab; 66 row tiles, i.e. three bands of row tiles (32, 32 and a ragged
+# 2) with a ragged last tile; one short of / one past the 128-row and 256-column tile edges with K off the
+# 64-column slab
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (200, 1000, 328), (384, 2304, 4096), (130, 151936, 64),
                                    (1, 8, 64), (257, 520, 72), (5, 40, 8), (8322, 1000, 64),
                                    (127, 255, 16), (129, 257, 136), (256, 512, 200), (255, 33, 24)])
@@ -95,7 +95,9 @@ def test_lmhead_matches_token_stats_on_same_logits():
 
 def test_lmhead_workload_full_chain():
     """32,768 tokens x 4,096 x 151,936: GEMM + merge, discrepancy, advantages,
-    controller, gradient on the stored logits; oracle on sampled rows."""
+    controller, gradient on the stored logits; the O(T) stages on every row,
+    the vocabulary-wide outputs on 1,024 random rows plus the first and last
+    row of every 128-row tile."""
     torch.cuda.empty_cache()
     b = W.generate_lmhead(device=DEV)
     p = acrl.Params()
@@ -124,33 +126,40 @@ def test_lmhead_workload_full_chain():
     ocoef = O.loss_coefficients(ow, oadv, mask, so, seq, grp, batch, op)
     tl_ref, loss_ref = O.surrogate_loss(host(logp).astype(np.float64), None, oadv, ow, mask, so, seq, grp, batch, op)
     assert_loss(float(loss), loss_ref, tl_ref)
-    # vocabulary-wide outputs on sampled rows, from the oracle's own fp64 logits
+    # vocabulary-wide outputs on sampled rows, from the oracle's own fp64 logits: 1,024 random rows and the first
+    # and last row of every 128-row tile (so every edge of the 32-tile bands too), in blocks of 256 rows
     rng = np.random.default_rng(3)
-    rows = np.unique(np.concatenate([rng.choice(b.T, size=40, replace=False), [0, b.T - 1]]))
+    starts = np.arange(0, b.T, 128)
+    rows = np.unique(np.concatenate([rng.choice(b.T, size=1024, replace=False), starts,
+                                     np.minimum(starts + 127, b.T - 1)]))
+    assert len(rows) >= 1024 + 2 * len(starts) - 64
     Wf = _f64(b.weight)
-    Hr = _f64(b.hidden[torch.as_tensor(rows, device=DEV)])
-    z = O.lmhead_logits(Hr, Wf)
-    abs_sum = np.abs(Hr) @ np.abs(Wf).T
-    del Wf
-    _check_logits(logits[torch.as_tensor(rows, device=DEV), :b.N], z, abs_sum, b.K, "logits (sampled rows)")
-    olse, ologp, oH, _ = O.token_stats(z, host(b.ids)[rows], mask[rows])
-    # a stored logit one bf16 ulp off the oracle's rounding (both valid) moves lse by p_j |dz_j| and log p by
-    # that plus |dz_a|: the statistics may differ from the oracle's chain by that much beyond TOL_LOGP
-    zg = rows_f64(logits, rows, b.N)
-    dz = np.abs(zg - z)
-    shift = (np.exp(z - olse[:, None]) * dz).sum(axis=1)
-    a = host(b.ids)[rows]
-    assert_close_abs(host(lse)[rows], olse, TOL_LOGP + shift, "lse")
-    assert_close_abs(host(logp)[rows], ologp, TOL_LOGP + shift + dz[np.arange(len(rows)), a], "logp")
-    assert_close_rel(host(ent)[rows], oH, floor=1e-5, what="entropy")
-    # The gradient pass is judged on the logits it consumed: a logit one bf16 ulp
-    # away (about 0.1 % of them, see _check_logits) moves its p by e^ulp, ~1-2 %.
-    glse, _, _, _ = O.token_stats(zg, host(b.ids)[rows], mask[rows])
-    lse_full = np.zeros(b.T)
-    lse_full[rows] = glse
-    ograd, _, _ = O.loss_grad_logits(zg, host(b.ids), mask, lse_full, None, oadv, ow, so, seq, grp, batch, op,
-                                     rows=rows)
-    assert_grad_rows(grad_rows(grad, rows, b.N), ograd, ocoef[rows], host(b.ids)[rows])
+    Wabs = np.abs(Wf)
+    ids_h = host(b.ids)
+    lse_h, logp_h, ent_h = host(lse), host(logp), host(ent)
+    for k in range(0, len(rows), 256):
+        rr = rows[k:k + 256]
+        Hr = _f64(b.hidden[torch.as_tensor(rr, device=DEV)])
+        z = O.lmhead_logits(Hr, Wf)
+        _check_logits(logits[torch.as_tensor(rr, device=DEV), :b.N], z, np.abs(Hr) @ Wabs.T, b.K,
+                      "logits (sampled rows)")
+        olse, ologp, oH, _ = O.token_stats(z, ids_h[rr], mask[rr])
+        # a stored logit one bf16 ulp off the oracle's rounding (both valid) moves lse by p_j |dz_j| and log p by
+        # that plus |dz_a|: the statistics may differ from the oracle's chain by that much beyond TOL_LOGP
+        zg = rows_f64(logits, rr, b.N)
+        dz = np.abs(zg - z)
+        shift = (np.exp(z - olse[:, None]) * dz).sum(axis=1)
+        a = ids_h[rr]
+        assert_close_abs(lse_h[rr], olse, TOL_LOGP + shift, "lse")
+        assert_close_abs(logp_h[rr], ologp, TOL_LOGP + shift + dz[np.arange(len(rr)), a], "logp")
+        assert_close_rel(ent_h[rr], oH, floor=1e-5, what="entropy")
+        # The gradient pass is judged on the logits it consumed: a logit one bf16 ulp
+        # away (about 0.1 % of them, see _check_logits) moves its p by e^ulp, ~1-2 %.
+        glse, _, _, _ = O.token_stats(zg, ids_h[rr], mask[rr])
+        lse_full = np.zeros(b.T)
+        lse_full[rr] = glse
+        ograd, _, _ = O.loss_grad_logits(zg, ids_h, mask, lse_full, None, oadv, ow, so, seq, grp, batch, op, rows=rr)
+        assert_grad_rows(grad_rows(grad, rr, b.N), ograd, ocoef[rr], a)
 
 
 def test_lmhead_flags_nonfinite_and_bad_id_rows_like_token_stats():
@@ -183,3 +192,62 @@ def test_lmhead_flags_nonfinite_and_bad_id_rows_like_token_stats():
     assert_close_abs(host(logp[ok]), host(logp2[ok]), 2e-5, "logp")
     assert_close_rel(host(ent[ok]), host(ent2[ok]), rel=1e-4, floor=1e-6, what="entropy")
     assert torch.isnan(lse2[5]) and float(logp2[7]) == 0.0
+
+
+def _managed_alloc(nbytes):
+    """Managed memory from the driver API (cuMemAllocManaged, attached
+    globally), for the operand-placement check; returns (address, free)."""
+    import ctypes
+    cu = ctypes.CDLL("libcuda.so.1")
+    torch.cuda.synchronize()              # the runtime has made the primary context current on this thread
+    p = ctypes.c_uint64(0)
+    assert cu.cuMemAllocManaged(ctypes.byref(p), ctypes.c_size_t(nbytes), ctypes.c_uint(1)) == 0 and p.value
+    return p.value, lambda: cu.cuMemFree_v2(ctypes.c_uint64(p.value))
+
+
+def test_lmhead_refuses_operands_outside_this_gpu():
+    """hidden, weight and logits must be plain device memory of the current
+    device, since the GEMM's TMA copies are encoded over them: managed memory
+    and host memory (page-locked or pageable) are refused on the host with
+    ACRL_ERR_INVALID_ARG before anything is launched, by both LM-head entry
+    points, and the context stays usable."""
+    M, N, K = 130, 264, 64
+    gen = torch.Generator(device=DEV).manual_seed(21)
+    H = torch.randn((M, K), generator=gen, device=DEV).to(torch.bfloat16)
+    Wt = (0.02 * torch.randn((N, K), generator=gen, device=DEV)).to(torch.bfloat16)
+    ids = torch.randint(0, N, (M,), generator=gen, device=DEV, dtype=torch.int32)
+    logits = torch.full((M, N), 7.0, dtype=torch.bfloat16, device=DEV)
+    partials = torch.empty(api.lmhead_workspace_bytes(M, N) // 4, dtype=torch.float32, device=DEV)
+    out = [torch.full((M,), 3.0, device=DEV) for _ in range(3)]
+    flags = api.new_flags()
+    L = _abi.lib()
+    stream = torch.cuda.current_stream().cuda_stream
+    size = max(M, N) * max(K, N) * 2
+    pinned = torch.empty(size // 2, dtype=torch.bfloat16, pin_memory=True)
+    pageable = torch.empty(size // 2, dtype=torch.bfloat16)
+    managed, free_managed = _managed_alloc(size)
+    try:
+        for bad in (managed, pinned.data_ptr(), pageable.data_ptr()):
+            assert bad % 16 == 0
+            for slot in range(3):
+                ptrs = [H.data_ptr(), Wt.data_ptr(), logits.data_ptr()]
+                ptrs[slot] = bad
+                st = L.acrl_lmhead_logits_stats(ptrs[0], M, K, K, ptrs[1], N, K, ptrs[2], N, partials.data_ptr(),
+                                                flags.data_ptr(), stream)
+                assert st == _abi.ERR_INVALID_ARG, (hex(bad), slot, st)
+                st = L.acrl_lmhead_stats_noalloc(ptrs[0], M, K, K, ptrs[1], N, K, ptrs[2], N, ids.data_ptr(), None,
+                                                 out[0].data_ptr(), out[1].data_ptr(), out[2].data_ptr(),
+                                                 flags.data_ptr(), stream)
+                assert st == _abi.ERR_INVALID_ARG, (hex(bad), slot, st)
+        torch.cuda.synchronize()
+        # nothing ran: outputs untouched, no flag raised
+        assert api.read_flags(flags) == 0
+        assert bool((logits.float() == 7.0).all()) and all(bool((t == 3.0).all()) for t in out)
+    finally:
+        free_managed()
+    # the same call on device memory runs, and the context is fine
+    lg, part = api.lmhead_logits_stats(H, Wt, N=N, flags=flags)
+    lse, logp, ent = api.lmhead_merge(part, lg, ids, None, N=N, flags=flags)
+    assert api.read_flags(flags) == 0
+    lse2, _, _ = api.token_stats(lg, ids, None, V=N)
+    assert_close_abs(host(lse), host(lse2), 1e-5, "lse after the refusals")

@@ -1,10 +1,11 @@
 """GPU parity at the full workload sizes, in the launch configuration the
 benchmark times.  The vocabulary-wide outputs (lse, logp, entropy, gradient)
-are checked on sampled rows: random valid rows, every row of two whole
-responses, and the first and last row of the batch (and of each chunk).  Every
-O(T) output is checked on all rows, stage-isolated: the oracle's discrepancy,
-advantage and controller stages are fed the GPU's fp32 log-probs.  The oracle's
-own full chain is checked on the sampled whole responses."""
+are checked element by element on sampled rows: 4,096 random valid rows,
+every row of 4 whole responses, the first and last row of the batch, and the
+first and last row of each gradient chunk.  Every O(T) output is checked on
+all rows, stage-isolated: the oracle's discrepancy, advantage and controller
+stages are fed the GPU's fp32 log-probs.  The oracle's own full chain (its
+log-softmax, then the discrepancy) is checked on the whole responses."""
 
 import numpy as np
 import pytest
@@ -12,8 +13,8 @@ import torch
 
 import oracle as O
 import workloads as W
-from parity import (TOL_LOGP, assert_close_abs, assert_close_rel, assert_grad_rows, assert_loss, compare_batch,
-                    compare_grp, compare_seq, grad_rows, host, oracle_params, rows_f64)
+from parity import (VocabRowCheck, assert_close_abs, assert_close_rel, assert_grad_rows, assert_loss, compare_batch,
+                    compare_grp, compare_seq, grad_rows, host, oracle_params)
 
 pytestmark = pytest.mark.gpu
 
@@ -23,7 +24,7 @@ from paper_2607_24062_gb300 import api  # noqa: E402
 DEV = "cuda"
 
 
-def _sample_rows(b, rng, n_random=384, n_whole=2, extra=()):
+def _sample_rows(b, rng, n_random=4096, n_whole=4, extra=()):
     mask = host(b.mask)
     so = host(b.seq_offsets)
     valid = np.flatnonzero(mask)
@@ -66,35 +67,25 @@ def _oracle_O_T(step, b, op):
     return dict(lr=lr, seq=seq, grp=grp, batch=batch, adv=adv, w=w, coef=coef)
 
 
-def _check_rows(step, b, rows, ref, op, grad=None, grad_row0=0, block=512):
-    """a1 and a6 on `rows` against the oracle's own fp64 log-softmax (in blocks
-    of rows to bound host memory)."""
-    ids, mask = host(b.ids), host(b.mask)
-    g = grad if grad is not None else step.grad
-    for k in range(0, len(rows), block):
-        rr = rows[k:k + block]
-        z = rows_f64(b.logits, rr, b.V)
-        olse, ologp, oH, f = O.token_stats(z, ids[rr], mask[rr])
-        assert f == 0
-        assert_close_abs(host(step.lse)[rr], olse, TOL_LOGP, "lse")
-        assert_close_abs(host(step.logp)[rr], ologp, TOL_LOGP, "logp")
-        assert_close_rel(host(step.entropy)[rr], oH, floor=1e-5, what="entropy")
-        lse_full = np.zeros(b.T)
-        lse_full[rr] = olse
-        ograd, otl, _ = O.loss_grad_logits(z, ids, mask, lse_full, None, ref["adv"], ref["w"],
-                                           host(b.seq_offsets), ref["seq"], ref["grp"], ref["batch"], op, rows=rr)
-        assert_grad_rows(grad_rows(g, rr - grad_row0, b.V), ograd, ref["coef"][rr], ids[rr])
+def _check_rows(step, b, rows, ref, op):
+    """a1 and a6 on `rows` against the oracle's own fp64 log-softmax and gradient (blocks of rows in the oracle
+    pool); returns the checker, which keeps the oracle's logp and entropy of those rows."""
+    chk = VocabRowCheck(b.T, host(b.ids), host(b.mask), host(b.seq_offsets), ref, op)
+    chk.submit(b.logits, b.V, rows, step.lse, step.logp, step.entropy, step.grad)
+    assert chk.finish() == len(rows)
+    return chk
 
 
-def _oracle_chain_on_whole(step, b, whole, op):
-    """The oracle's own chain (its log-softmax, then the discrepancy) on whole responses."""
+def _oracle_chain_on_whole(step, b, whole, chk):
+    """The oracle's own chain (its log-softmax, then the discrepancy) on whole responses; the oracle's log-probs
+    and entropies are those the row check computed."""
     so, mask = host(b.seq_offsets), host(b.mask)
     mu = host(b.logp_mu).astype(np.float64)
     gseq = step.seq_host()
     for i in whole:
         r = np.arange(int(so[i]), int(so[i + 1]))
-        z = rows_f64(b.logits, r, b.V)
-        _, ologp, oH, _ = O.token_stats(z, host(b.ids)[r], mask[r])
+        ologp = np.array([chk.oracle_logp[t] for t in r.tolist()])
+        oH = np.array([chk.oracle_entropy[t] for t in r.tolist()])
         lr, d, seq, _, _, _ = O.seq_discrepancy(ologp, mu[r], mask[r], [0, len(r)], [0, 1], oH)
         assert int(gseq["n"][i]) == int(seq["n"][0])
         assert_close_rel(gseq["mean_d"][i], seq["mean_d"][0], floor=1e-7, what=f"D_{i} (oracle chain)")
@@ -116,8 +107,8 @@ def test_full_size_workload(name):
     ref = _oracle_O_T(step, b, op)
     rng = np.random.default_rng(11)
     rows, whole = _sample_rows(b, rng)
-    _check_rows(step, b, rows, ref, op)
-    _oracle_chain_on_whole(step, b, whole, op)
+    chk = _check_rows(step, b, rows, ref, op)
+    _oracle_chain_on_whole(step, b, whole, chk)
     # cached-old path (lse recomputed inside the gradient call by a first sweep over each row) on the first
     # 4,096 rows: the same gradient as the streaming call
     R = min(4096, b.T)
@@ -175,19 +166,23 @@ def test_long_workload_chunked():
     assert_close_rel(host(step.coef), coef, floor=1e-12, what="coef")
     ref = dict(seq=seq, grp=grp, batch=batch, adv=adv, w=w, coef=coef)
     rng = np.random.default_rng(5)
-    rows_all, _ = _sample_rows(b, rng, n_random=256, n_whole=0)
+    rows_all, whole = _sample_rows(b, rng)
+    chk = VocabRowCheck(b.T, host(b.ids), mask, so, ref, op)
     checked = []
 
     def on_chunk(r0, r1, g):
+        # the chunk buffer is reused for the next chunk: the rows are copied out before this returns
         torch.cuda.synchronize()
         rows = rows_all[(rows_all >= r0) & (rows_all < r1)]
         rows = np.unique(np.concatenate([rows, [r0, r1 - 1]]))
-        _check_rows(step, b, rows, ref, op, grad=g, grad_row0=r0)
+        chk.submit(b.logits, b.V, rows, step.lse, step.logp, step.entropy, grad=g, grad_row0=r0)
         checked.append(len(rows))
 
     step.gradient(b.logits, b.ids, b.mask, chunk_rows=spec.chunk_rows, on_chunk=on_chunk)
     torch.cuda.synchronize()
-    assert sum(checked) >= len(rows_all) and len(checked) == (b.T + spec.chunk_rows - 1) // spec.chunk_rows
+    assert chk.finish() == sum(checked) >= len(rows_all)
+    assert len(checked) == (b.T + spec.chunk_rows - 1) // spec.chunk_rows
+    _oracle_chain_on_whole(step, b, whole, chk)
     tl, loss = O.surrogate_loss(lp, None, adv, w, mask, so, seq, grp, batch, op)
     assert_close_rel(host(step.token_loss), tl, floor=1e-12, what="token_loss")
     assert_loss(float(step.loss), loss, tl)
