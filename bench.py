@@ -162,6 +162,19 @@ def _lmhead_desc(b):
             "mu from E4M3 per-token/per-channel copies")
 
 
+def _logits_config(spec, batch, world):
+    """`config` of a logits workload's line; both arms print the same one."""
+    return {"workload": _workload_desc(spec), "T": batch.T, "V": batch.V, "ld": batch.ld,
+            "tokens_per_step": int(batch.mask.sum()), "logits": "bf16 in, gradient bf16 out, fp32 arithmetic",
+            "l2": f"no flush: inputs ({batch.T * batch.ld * 2 / 1e9:.1f} GB of logits) far larger than the 129 MB L2",
+            "parallelism": f"data-parallel over prompts, {world} rank(s); 3-scalar all-reduce per step"}
+
+
+def _lmhead_config(b):
+    """`config` of the LM-head workload's line; both arms print the same one."""
+    return {"workload": _lmhead_desc(b), "M": b.T, "N": b.N, "K": b.K, "tokens_per_step": int(b.mask.sum())}
+
+
 def _workload_desc(spec):
     return (f"{spec.name}: {spec.n_prompts} prompts x {spec.group_size} responses, lengths U[{spec.len_lo},"
             f"{spec.len_hi}], V={spec.V}, bf16 logits {spec.dist}(scale {spec.scale}), mu = FP8-E4M3 "
@@ -348,11 +361,11 @@ def run_reference(args):
     if lmhead:
         spec = _lmhead_spec(W, args.workload)
         batch = W.generate_lmhead(spec, device=dev)
-        config = {"workload": _lmhead_desc(batch), "M": batch.T, "N": batch.N, "K": batch.K}
+        config = _lmhead_config(batch)
     else:
         spec = W.SPECS[args.workload]
         batch = W.generate(spec, seed=W.seed_for(spec.name), device=dev)
-        config = {"workload": _workload_desc(spec), "T": batch.T, "V": batch.V}
+        config = _logits_config(spec, batch, world)
     params = acrl.Params()
     vals = []
     t_all = []
@@ -538,10 +551,7 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic",
-        "config": {"workload": _workload_desc(spec), "T": batch.T, "V": V, "ld": batch.ld,
-                   "tokens_per_step": n_valid, "logits": "bf16 in, gradient bf16 out, fp32 arithmetic",
-                   "l2": "no flush: inputs (44.8 GB of logits) far larger than the 129 MB L2",
-                   "parallelism": f"data-parallel over prompts, {world} rank(s); 3-scalar all-reduce per step"},
+        "config": _logits_config(spec, batch, world),
         "roofline": {"bound": "hbm", "kernel": "acrl_loss_grad_logits", "achieved": k5_gbs, "peak": peak,
                      "unit": "GB/s", "frac": k5_gbs / peak, "traffic": traffic, "peak_kind": peak_kind,
                      "algorithmic_bytes_per_launch": k5_bytes, "ms_per_launch": k5_avg},
@@ -570,6 +580,16 @@ def run_ours(args):
         v, desc, n, cores = oracle_tokens_per_s(batch, params, rows_budget_s=args.ref_seconds, max_rows=16384)
         out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
                                "cpu": _cpu_model()}
+    if not args.no_lmhead and world == 1:
+        # The fused LM-head workload (hidden 32,768 x 4,096, weight 151,936 x 4,096) in the same process, once
+        # the Qwen batch's buffers are released: its own K steps after W warm-up steps, its own clock record.
+        # Reported beside the step above; the line's value, timing and launch count are the Qwen step's.
+        import gc
+        del step, batch, ent_coef
+        gc.collect()
+        torch.cuda.empty_cache()
+        lm, _, _ = lmhead_measure("lmhead", dev, args.steps, args.warmup)
+        out["kernels"]["lmhead_step (fused LM-head workload)"] = lm
     print(json.dumps(out))
     return 0
 
@@ -596,31 +616,28 @@ def _weight_calls_ms(acrl, W, dev, median_ms):
             "note": "includes the output allocations of the Python calls; the paper's 0.059 s is context only"}
 
 
-def _peak_tflops():
+def _tensor_peaks():
+    """Measured bf16 tensor throughput (TFLOP/s): (burst, sustained, kind)."""
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
         with open(path) as f:
             d = json.load(f)
-        return float(d["bf16_tflops_sustained"]), "measured (sustained)"
+        return float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
     except Exception:
-        return 1700.0, "fallback (sustained)"
+        return 1900.0, 1700.0, "fallback"
 
 
-def run_lmhead(args):
-    """The fused LM-head workload: 32,768 tokens x 4,096 hidden x 151,936
-    vocabulary.  A step is the GEMM with the statistics epilogue, the merge,
-    the O(T) stages and the gradient on the stored bf16 logits."""
+def lmhead_measure(workload, dev, steps, warmup):
+    """Time the fused LM-head workload (32,768 tokens x 4,096 hidden x 151,936
+    vocabulary for "lmhead"): a step is the GEMM with the statistics epilogue,
+    the merge, the O(T) stages and the gradient on the stored bf16 logits,
+    every call through the C ABI.  Returns (summary dict, batch, params)."""
     import torch
 
     import paper_2607_24062_gb300 as acrl
     import workloads as W
-    from paper_2607_24062_gb300 import build
 
-    world, rank, local = _dist()
-    build.build()
-    dev = torch.device(f"cuda:{local}")
-    torch.cuda.set_device(dev)
-    b = W.generate_lmhead(_lmhead_spec(W, args.workload), device=dev)
+    b = W.generate_lmhead(_lmhead_spec(W, workload), device=dev)
     p = acrl.Params()
     M, N, K = b.T, b.N, b.K
     stream = torch.cuda.current_stream(dev)
@@ -652,15 +669,15 @@ def run_lmhead(args):
         if ev:
             ev[4].record(stream)
 
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         one()
     torch.cuda.synchronize()
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(dev.index) as clocks:
         torch.cuda.synchronize()
         t0.record(stream)
-        for k in range(args.steps):
+        for k in range(steps):
             one(evs[k])
         t1.record(stream)
         torch.cuda.synchronize()
@@ -668,25 +685,54 @@ def run_lmhead(args):
     total_ms = t0.elapsed_time(t1)
     gemm_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in evs]))
     merge_ms = float(np.mean([e[1].elapsed_time(e[2]) for e in evs]))
+    ot_ms = float(np.mean([e[2].elapsed_time(e[3]) for e in evs]))
     grad_ms = float(np.mean([e[3].elapsed_time(e[4]) for e in evs]))
     flop = 2.0 * M * N * K
     tf = flop / (gemm_ms / 1e3) / 1e12
-    peak, kind = _peak_tflops()
+    burst, sustained, kind = _tensor_peaks()
     n_valid = int(b.mask.sum())
+    ms_step = total_ms / steps
+    summary = {
+        "workload": _lmhead_desc(b), "M": M, "N": N, "K": K, "steps": steps, "warmup": warmup, "flags": fl,
+        "ms_per_step": ms_step, "tokens/s": n_valid / (ms_step / 1e3), "tokens_per_step": n_valid,
+        "gemm": {"kernel": "acrl_lmhead_logits_stats", "ms": gemm_ms, "TFLOP/s": tf, "flop_per_launch": flop,
+                 "frac_burst": tf / burst, "frac_sustained": tf / sustained, "peak_burst": burst,
+                 "peak_sustained": sustained, "peak_kind": kind},
+        "merge_ms": merge_ms, "seq_discrepancy+grpo_advantage+controller_step_ms": ot_ms,
+        "loss_grad_logits": {"ms": grad_ms, "GB/s": 4.0 * M * N / (grad_ms / 1e3) / 1e9},
+        "clocks": clocks.summary(), "gpu_launches": 10 * steps,
+    }
+    return summary, b, p
+
+
+def run_lmhead(args):
+    """The fused LM-head workload on its own line (`--workload lmhead` or
+    `lmhead_profile`)."""
+    import torch
+
+    from paper_2607_24062_gb300 import build
+
+    world, rank, local = _dist()
+    build.build()
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    lm, b, p = lmhead_measure(args.workload, dev, args.steps, args.warmup)
+    g = lm["gemm"]
     out = {"metric": LMHEAD_METRIC,
-           "value": n_valid * args.steps / (total_ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
-           "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+           "value": lm["tokens/s"], "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": lm["ms_per_step"], "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "bf16 (tensor cores, fp32 accumulate)", "data": "synthetic",
-           "config": {"workload": _lmhead_desc(b), "flags": fl},
-           "roofline": {"bound": "tensor", "kernel": "acrl_lmhead_logits_stats", "achieved": tf, "peak": peak,
-                        "unit": "TFLOP/s", "frac": tf / peak,
+           "config": _lmhead_config(b), "device_flags": lm["flags"],
+           "roofline": {"bound": "tensor", "kernel": g["kernel"], "achieved": g["TFLOP/s"],
+                        "peak": g["peak_sustained"], "unit": "TFLOP/s", "frac": g["frac_sustained"],
+                        "frac_burst": g["frac_burst"], "peak_burst": g["peak_burst"],
                         "traffic": _traffic_of("lmhead.cu") if args.workload == "lmhead" else None,
-                        "peak_kind": kind, "flop_per_launch": flop, "ms_per_launch": gemm_ms},
-           "kernels": {"acrl_lmhead_logits_stats": {"ms": gemm_ms, "TFLOP/s": tf},
-                       "acrl_lmhead_merge": {"ms": merge_ms},
-                       "acrl_loss_grad_logits": {"ms": grad_ms,
-                                                 "GB/s": 4.0 * M * N / (grad_ms / 1e3) / 1e9}},
-           "clocks": clocks.summary(), "gpu_launches": 10 * args.steps}
+                        "peak_kind": g["peak_kind"] + " (sustained)", "flop_per_launch": g["flop_per_launch"],
+                        "ms_per_launch": g["ms"]},
+           "kernels": {"acrl_lmhead_logits_stats": {"ms": g["ms"], "TFLOP/s": g["TFLOP/s"]},
+                       "acrl_lmhead_merge": {"ms": lm["merge_ms"]},
+                       "acrl_loss_grad_logits": lm["loss_grad_logits"]},
+           "clocks": lm["clocks"], "gpu_launches": lm["gpu_launches"]}
     if not args.no_cpu:
         v, desc, _, cores = oracle_tokens_per_s(b, p, rows_budget_s=args.ref_seconds, lmhead=True)
         out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
@@ -848,6 +894,8 @@ def main():
     ap.add_argument("--e2e-chunks", type=int, default=16)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-lmhead", action="store_true",
+                    help="skip the fused LM-head workload that the default run times after the Qwen step")
     ap.add_argument("--ref-seconds", type=float, default=10.0)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":

@@ -22,6 +22,12 @@ def test_reference_arm_prints_one_json_line():
     assert out["impl"] == "reference" and out["unit"] == "tokens/s" and out["higher_is_better"] is True
     assert out["value"] > 0 and out["steps"] == 2 and out["warmup"] == 1
     assert out["config"]["workload"].startswith("tiny")
+    # the same config, key for key, as the repository's own arm prints for this workload
+    sys.path.insert(0, ROOT)
+    import bench
+    import workloads as W
+    spec = W.SPECS["tiny"]
+    assert out["config"] == bench._logits_config(spec, W.generate(spec, seed=W.seed_for(spec.name)), 1)
     cb = out["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == out["value"] and "sampled rows" in cb["sample"]
     assert cb["cores"] == len(os.sched_getaffinity(0)) or cb["cores"] == 32

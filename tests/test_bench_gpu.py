@@ -37,3 +37,10 @@ def test_bench_line_has_the_contract_keys():
     cb = out["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] > 0
     assert set(out["clocks"]) >= {"sm_mhz", "sm_max_mhz", "reasons"}
+    # the fused LM-head workload, timed in the same process after the logits step
+    lm = out["kernels"]["lmhead_step (fused LM-head workload)"]
+    assert (lm["M"], lm["N"], lm["K"], lm["flags"], lm["steps"]) == (32768, 151936, 4096, 0, 3)
+    g = lm["gemm"]
+    assert g["TFLOP/s"] > 0 and g["frac_burst"] == pytest.approx(g["TFLOP/s"] / g["peak_burst"])
+    assert g["frac_sustained"] == pytest.approx(g["TFLOP/s"] / g["peak_sustained"])
+    assert set(lm["clocks"]) >= {"sm_mhz", "sm_max_mhz", "reasons"}
