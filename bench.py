@@ -46,14 +46,18 @@ FALLBACK_HBM_GBS = 6800.0
 # Kernel launches per step inside the timed region: token_stats 1, seq_discrepancy 2,
 # grpo_advantage 1, controller_step 3, loss_grad_logits 2.
 LAUNCHES_PER_STEP = 9
-# DRAM traffic of one launch of each kernel on its bench workload, from ncu
-# (dram__bytes_read.sum + dram__bytes_write.sum, one pass), valid only for the kernel
-# source it was taken on (sha256 of the file and the headers beside it, first 16 hex digits).
+# DRAM traffic of one launch of each kernel (dram__bytes_read.sum + dram__bytes_write.sum
+# from ncu, one pass), captured on a small case of its workload and scaled to a full
+# launch by the algorithmic bytes (or, for the GEMM, the flops) of each: the streaming
+# kernels' traffic grows in proportion to the rows, the GEMM's to the bands of 32 row
+# tiles (the weight is read once per band).  Valid only for the kernel source it was
+# taken on (sha256 of the file and the headers beside it, first 16 hex digits).
 NCU_TRAFFIC = {
-    "loss_grad.cu": {"src": "fabc7049c1e852c1", "bytes_per_launch": 41.71e9 + 44.87e9},
-    "token_stats.cu": {"src": "4100be30fb1483c9", "bytes_per_launch": 44.94e9 + 3.75e6},
-    # the LM-head GEMM at 32,768 x 4,096 x 151,936
-    "lmhead.cu": {"src": "463e708e245c83b1", "bytes_per_launch": 11.93e9 + 10.35e9},
+    # qwen_profile (8,192 rows x 151,936), the two timed launches averaged
+    "loss_grad.cu": {"src": "d8782a0747bda5ba", "bytes": 2.4896e9 + 2.4371e9, "units": 4978778112},
+    "token_stats.cu": {"src": "d1643f8219277aa2", "bytes": 2.49025e9 + 1.65e6, "units": 2489458688},
+    # lmhead_profile (4,096 x 4,096 x 151,936: one band), flops as the unit
+    "lmhead.cu": {"src": "a8604f527150f0a7", "bytes": 2.1415e9 + 1.3065e9, "units": 2.0 * 4096 * 151936 * 4096},
 }
 
 
@@ -78,10 +82,15 @@ def _src_hash(name):
     return d.hexdigest()[:16]
 
 
-def _traffic_of(name):
-    """ncu DRAM bytes per launch of a kernel source, if taken on the source as it is now."""
+TRAFFIC_SOURCE = ("ncu dram__bytes_read.sum + dram__bytes_write.sum on a small case (qwen_profile, 8,192 rows; "
+                  "lmhead_profile, 4,096 rows) scaled by algorithmic bytes (flops for the GEMM)")
+
+
+def _traffic_of(name, units):
+    """ncu DRAM bytes per launch of a kernel source scaled to a launch of `units`
+    algorithmic bytes (flops for the GEMM), if taken on the source as it is now."""
     tr = NCU_TRAFFIC.get(name)
-    return tr["bytes_per_launch"] if tr and tr["src"] == _src_hash(name) else None
+    return tr["bytes"] * units / tr["units"] if tr and tr["src"] == _src_hash(name) else None
 
 
 class ClockSampler:
@@ -514,7 +523,7 @@ def run_ours(args):
     k1_avg = float(np.mean(k1_ms))
     k5_gbs = k5_bytes / (k5_avg / 1e3) / 1e9
     k1_gbs = k1_bytes / (k1_avg / 1e3) / 1e9
-    traffic = _traffic_of("loss_grad.cu")
+    traffic = _traffic_of("loss_grad.cu", k5_bytes)
 
     # the same step replayed from a CUDA graph (launch gaps removed); reported beside the eager step
     # (single process only: the multi-rank step keeps its collective outside any graph)
@@ -554,10 +563,11 @@ def run_ours(args):
         "config": _logits_config(spec, batch, world),
         "roofline": {"bound": "hbm", "kernel": "acrl_loss_grad_logits", "achieved": k5_gbs, "peak": peak,
                      "unit": "GB/s", "frac": k5_gbs / peak, "traffic": traffic, "peak_kind": peak_kind,
-                     "algorithmic_bytes_per_launch": k5_bytes, "ms_per_launch": k5_avg},
+                     "traffic_source": TRAFFIC_SOURCE, "algorithmic_bytes_per_launch": k5_bytes,
+                     "ms_per_launch": k5_avg},
         "kernels": {
             "acrl_token_stats": {"ms": k1_avg, "GB/s": k1_gbs, "frac": k1_gbs / peak, "bytes": k1_bytes,
-                                 "traffic": _traffic_of("token_stats.cu")},
+                                 "traffic": _traffic_of("token_stats.cu", k1_bytes)},
             "acrl_loss_grad_logits": {"ms": k5_avg, "GB/s": k5_gbs, "frac": k5_gbs / peak, "bytes": k5_bytes},
             "seq_discrepancy+grpo_advantage+controller_step": {"ms": float(np.mean(mid_ms))},
             "acrl_loss_grad_logits (lse recomputed, cached-old)": {
@@ -697,7 +707,8 @@ def lmhead_measure(workload, dev, steps, warmup):
         "ms_per_step": ms_step, "tokens/s": n_valid / (ms_step / 1e3), "tokens_per_step": n_valid,
         "gemm": {"kernel": "acrl_lmhead_logits_stats", "ms": gemm_ms, "TFLOP/s": tf, "flop_per_launch": flop,
                  "frac_burst": tf / burst, "frac_sustained": tf / sustained, "peak_burst": burst,
-                 "peak_sustained": sustained, "peak_kind": kind},
+                 "peak_sustained": sustained, "peak_kind": kind, "traffic": _traffic_of("lmhead.cu", flop),
+                 "traffic_source": TRAFFIC_SOURCE},
         "merge_ms": merge_ms, "seq_discrepancy+grpo_advantage+controller_step_ms": ot_ms,
         "loss_grad_logits": {"ms": grad_ms, "GB/s": 4.0 * M * N / (grad_ms / 1e3) / 1e9},
         "clocks": clocks.summary(), "gpu_launches": 10 * steps,
@@ -726,7 +737,7 @@ def run_lmhead(args):
            "roofline": {"bound": "tensor", "kernel": g["kernel"], "achieved": g["TFLOP/s"],
                         "peak": g["peak_sustained"], "unit": "TFLOP/s", "frac": g["frac_sustained"],
                         "frac_burst": g["frac_burst"], "peak_burst": g["peak_burst"],
-                        "traffic": _traffic_of("lmhead.cu") if args.workload == "lmhead" else None,
+                        "traffic": _traffic_of("lmhead.cu", g["flop_per_launch"]),
                         "peak_kind": g["peak_kind"] + " (sustained)", "flop_per_launch": g["flop_per_launch"],
                         "ms_per_launch": g["ms"]},
            "kernels": {"acrl_lmhead_logits_stats": {"ms": g["ms"], "TFLOP/s": g["TFLOP/s"]},

@@ -5,24 +5,35 @@
 // lse, the sampled token's log-prob and the entropy without reading the logits
 // again.
 //
-// Blackwell path: a persistent kernel, one CTA per SM, warp-specialised.
-//   warp 0     one thread issues TMA tile loads (128B-swizzled) into a 4-stage
-//              shared-memory ring of A 128x64 + B 256x64 bf16;
-//   warp 1     one thread issues tcgen05.mma (M=128, N=256, K=16, kind::f16)
-//              into a TMEM accumulator and commits each stage back to the
-//              producer; two 256-column accumulators alternate between tiles;
-//   warps 2-5  the epilogue: tcgen05.ld of the accumulator (each thread one
-//              row), round to bf16, fold the statistics, and write the logits
-//              through shared memory with TMA bulk tensor stores (32 x 32
-//              blocks, two staging buffers per warp).
-// Tiles are visited in bands of 32 row tiles so that the weight tiles in
-// flight are shared through L2 by the CTAs working on the same band.  Every
-// CTA loads its operands from this GPU's memory into its own shared memory
-// only (the tensor maps are encoded over pointers that the entry points have
-// checked to be device memory of the current device).
+// Blackwell path: a persistent kernel of CTA pairs (clusters of two CTAs,
+// tcgen05 cta_group::2), one CTA per SM, warp-specialised.  A pair computes a
+// 256 x 256 tile of the logits: each CTA stages its own 128 rows of H and its
+// 128-row half of the weight tile, and the MMAs of the even CTA read both
+// CTAs' shared memory and write each CTA's 128 accumulator rows into that
+// CTA's TMEM.  Per SM a K slab is 32 KB (A 128 x 64 + B 128 x 64), so six
+// stages fit and the weight half is never staged twice in a pair.
+//   warp 0     in each CTA, one thread issues the TMA loads (128B-swizzled)
+//              of the CTA's A and B into a 6-stage ring, counted on the even
+//              CTA's stage barrier;
+//   warp 1     in the even CTA, one thread issues tcgen05.mma (M=256, N=256,
+//              K=16, kind::f16) into one of two 256-column accumulators and
+//              releases each stage to the producers of both CTAs, one commit
+//              per CTA;
+//   warps 2-5  in each CTA, the epilogue: tcgen05.ld of its accumulator rows
+//              (each thread one row), round to bf16, fold the statistics, and
+//              write the logits through shared memory with TMA bulk tensor
+//              stores (32 x 32 blocks, two staging buffers per warp).
+// Tiles are visited in bands of 32 row tiles (16 pairs) so that the weight
+// tiles in flight are shared through L2 by the pairs working on the same band.
+// Every CTA loads only from this GPU's memory into its own shared memory (the
+// tensor maps are encoded over pointers that the entry points have checked to
+// be device memory of the current device), and each load fills that CTA's
+// shared memory alone.
 // Every wait on an mbarrier is bounded in time; on expiry the kernel raises
 // ACRL_FLAG_TIMEOUT, lets the copies it issued land, and exits after freeing
-// its TMEM.
+// its TMEM.  The two CTAs meet at a cluster barrier after initialising their
+// barriers and again before either frees its TMEM or exits, so neither touches
+// a peer that has gone.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -36,67 +47,78 @@
 namespace acrl {
 namespace {
 
-constexpr int kBM = 128, kBN = 256;
+constexpr int kBM = 128, kBN = 256;   // rows of H per CTA, columns (weight rows) per tile
+constexpr int kBK = 64;               // K slab: 64 bf16 = one 128-byte row under the 128-byte swizzle
+constexpr int kStages = 6;
+constexpr int kHalfBN = kBN / 2;      // weight rows staged by each CTA of a pair
+constexpr int kABytes = kBM * kBK * 2;
+constexpr int kBBytes = kHalfBN * kBK * 2;
+constexpr int kStageBytes = kABytes + kBBytes;   // per CTA; the pair's stage barrier counts twice this
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
-constexpr int kBandM = 32;
+constexpr int kBandM = 32;            // row tiles per band (16 pairs)
 // Output staging: each epilogue warp owns two 32 x 32 bf16 blocks (its 32
 // rows x one 32-column chunk of the accumulator), stored 64-byte-swizzled.
 constexpr int kOutBlockBytes = 32 * 32 * 2;
 constexpr int kOutBytes = 4 * 2 * kOutBlockBytes;
-// Instruction descriptor of tcgen05.mma kind::f16: D f32 (bits 4-5 = 1),
-// A and B bf16 (bits 7-9, 10-12 = 1), both K-major, N/8 at bit 17, M/16 at bit 24.
+// Instruction descriptor of tcgen05.mma kind::f16: D f32 (bits 4-5 = 1), A and
+// B bf16 (bits 7-9, 10-12 = 1), both K-major, N/8 at bit 17, M/16 at bit 24
+// (M = 256 across the pair, 128 rows in each CTA's TMEM).
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kBN >> 3) << 17) |
-                            (uint32_t(kBM >> 4) << 24);
-
-// Shape of the shared-memory ring: K-slab width BK (64 columns = 128-byte
-// rows under the 128-byte swizzle, 32 columns = 64-byte rows under the 64-byte
-// swizzle) and the number of stages.  The loads in flight cover (STAGES - 1)
-// stages of MMA time.  Measured on 32768 x 4096 x 151936: 64 x 4 stages 1574
-// TFLOP/s, 64 x 3 1439; 32 x 6, 8 or 9 stages 1056-1171 whatever the depth (the
-// operand reads of 64-byte-swizzled tiles are the limit there).  A fifth
-// 64-column stage does not fit in shared memory.
-template <int BK, int STAGES>
-struct Ring {
-    static_assert(BK == 32 || BK == 64, "K slab of 32 or 64 bf16 columns");
-    static constexpr int kBK = BK, kStages = STAGES;
-    static constexpr int kRowBytes = BK * 2;
-    static constexpr int kABytes = kBM * kRowBytes;
-    static constexpr int kBBytes = kBN * kRowBytes;
-    static constexpr int kStageBytes = kABytes + kBBytes;
-    // tcgen05 shared-memory descriptor: swizzle code (2 = 128-byte, 4 = 64-byte)
-    // and the stride between 8-row groups
-    static constexpr uint64_t kSwizzleCode = BK == 64 ? 2 : 4;
-    static constexpr uint32_t kGroupStride = 8 * kRowBytes;
-    static constexpr CUtensorMapSwizzle kTmaSwizzle = BK == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
-    struct Barriers {
-        uint64_t full[STAGES];
-        uint64_t empty[STAGES];
-        uint64_t tfull[2];
-        uint64_t tempty[2];
-        uint64_t mma_done;
-        uint32_t tmem_base;
-        int32_t abort;
-    };
-    // The B stages come first, then the A stages, the output staging blocks
-    // and the barriers, with a margin behind them (every descriptor read stays
-    // inside the allocation).
-    static constexpr int kMargin = 8192;
-    static constexpr int kSmemBytes = 1024 + STAGES * kStageBytes + kOutBytes + int(sizeof(Barriers)) + kMargin;
-    static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
+                            (uint32_t((2 * kBM) >> 4) << 24);
+// Barriers:
+//   full[s]    even CTA: both CTAs' copies of stage s landed
+//   empty[s]   each CTA: the MMAs reading stage s are done
+//   tfull[b]   each CTA: accumulator b is complete
+//   tempty[b]  even CTA: the eight epilogue warps of the pair drained accumulator b
+struct Barriers {
+    uint64_t full[kStages];
+    uint64_t empty[kStages];
+    uint64_t tfull[2];
+    uint64_t tempty[2];
+    uint64_t mma_done;
+    uint32_t tmem_base;
+    int32_t abort;
 };
-
-using LmRing = Ring<64, 4>;
+// The B stages come first, then the A stages, the output staging blocks and
+// the barriers, with a margin behind them (every descriptor read stays inside
+// the allocation).
+constexpr int kMargin = 8192;
+constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kOutBytes + int(sizeof(Barriers)) + kMargin;
+static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
 
 // ---------------------------------------------------------------------------
 // PTX wrappers
 // ---------------------------------------------------------------------------
 
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t peer_addr(const void* p, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+    return r;
+}
+
+__device__ __forceinline__ void remote_arrive(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// Tile load into this CTA's shared memory whose completion is counted on the
+// barrier at `bar` (a shared::cluster address: either CTA of the pair).
+__device__ __forceinline__ void tma_load_pair(void* dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
     asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-            smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+        "%3}], [%4];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
         : "memory");
 }
 
@@ -104,26 +126,26 @@ __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence:
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
 // Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with
-// the ring's swizzle: rows of BK*2 bytes, 8-row groups 8*BK*2 bytes apart.
-template <class R>
+// the 128-byte swizzle: rows of 128 bytes, 8-row groups 1024 bytes apart.
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
-    uint64_t d = uint64_t((addr & 0x3FFFFu) >> 4);            // start address
-    d |= uint64_t(R::kGroupStride >> 4) << 32;                 // stride between 8-row groups
-    d |= uint64_t(1) << 46;                                    // descriptor version of tcgen05
-    d |= R::kSwizzleCode << 61;                                // swizzle mode
+    uint64_t d = uint64_t((addr & 0x3FFFFu) >> 4);  // start address
+    d |= uint64_t(1024 >> 4) << 32;                  // stride between 8-row groups
+    d |= uint64_t(1) << 46;                          // descriptor version of tcgen05
+    d |= uint64_t(2) << 61;                          // 128-byte swizzle
     return d;
 }
 
-__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+__device__ __forceinline__ void mma_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
     asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
             tmem_d),
         "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate));
 }
 
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
-                 : "memory");
+// Arrive once on the barrier at shared::cluster address `bar` when this
+// thread's MMAs so far have completed.
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
 }
 
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
@@ -163,16 +185,17 @@ __device__ __forceinline__ void bulk_wait_read() {
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // ---------------------------------------------------------------------------
-// tile schedule: bands of BAND row tiles, all column tiles of a band in turn
+// tile schedule: bands of BAND row-tile pairs, all column tiles of a band in
+// turn; the pair of cluster c takes tiles c, c + clusters, ...
 // ---------------------------------------------------------------------------
 
-template <int BAND = kBandM>
-__device__ __forceinline__ void tile_coords(int t, int m_tiles, int n_tiles, int& m, int& n) {
+__device__ __forceinline__ void tile_coords(int t, int m_pairs, int n_tiles, int& mp, int& n) {
+    constexpr int BAND = kBandM / 2;
     const int per_band = BAND * n_tiles;
     const int band = t / per_band;
     const int r = t - band * per_band;
-    const int bm = min(BAND, m_tiles - band * BAND);
-    m = band * BAND + r % bm;
+    const int bm = min(BAND, m_pairs - band * BAND);
+    mp = band * BAND + r % bm;
     n = r / bm;
 }
 
@@ -185,18 +208,18 @@ __device__ __forceinline__ void give_up(volatile int32_t* abort, int32_t* flags)
 // roles
 // ---------------------------------------------------------------------------
 
-template <class R>
-__device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t* sA, uint8_t* sB,
-                         typename R::Barriers* bars, int m_tiles, int n_tiles, int total, int k_iters, int32_t* flags) {
-    constexpr int kStages = R::kStages;
+__device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t* sA, uint8_t* sB, Barriers* bars,
+                         uint32_t rank, int m_pairs, int n_tiles, int total, int k_iters, int32_t* flags) {
     volatile int32_t* abort = &bars->abort;
+    const int cl = int(blockIdx.x >> 1), ncl = int(gridDim.x >> 1);
     int stage = 0;
     uint32_t phase = 0;
     long issued = 0;
     bool ok = true;
-    for (int t = int(blockIdx.x); t < total && ok; t += int(gridDim.x)) {
-        int m, n;
-        tile_coords(t, m_tiles, n_tiles, m, n);
+    for (int t = cl; t < total && ok; t += ncl) {
+        int mp, n;
+        tile_coords(t, m_pairs, n_tiles, mp, n);
+        const int m = 2 * mp + int(rank);
         for (int kk = 0; kk < k_iters; ++kk) {
             if (!mbar_try_wait(&bars->empty[stage], phase ^ 1u) &&
                 !wait_phase(&bars->empty[stage], phase ^ 1u, abort)) {
@@ -204,9 +227,11 @@ __device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t
                 ok = false;
                 break;
             }
-            mbar_expect_tx(&bars->full[stage], R::kStageBytes);
-            tma_load_2d(sA + stage * R::kABytes, tmA, &bars->full[stage], kk * R::kBK, m * kBM);
-            tma_load_2d(sB + stage * R::kBBytes, tmB, &bars->full[stage], kk * R::kBK, n * kBN);
+            // the even CTA's barrier counts both CTAs' bytes of this stage
+            if (rank == 0) mbar_expect_tx(&bars->full[stage], 2 * kStageBytes);
+            const uint32_t full0 = peer_addr(&bars->full[stage], 0);
+            tma_load_pair(sA + stage * kABytes, tmA, full0, kk * kBK, m * kBM);
+            tma_load_pair(sB + stage * kBBytes, tmB, full0, kk * kBK, n * kBN + int(rank) * kHalfBN);
             ++issued;
             if (++stage == kStages) {
                 stage = 0;
@@ -215,25 +240,32 @@ __device__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, uint8_t
         }
     }
     if (!ok) {
-        // let the copies this thread started land before the CTA can exit
-        for (long j = issued - 1; j >= 0 && j >= issued - kStages; --j)
-            wait_phase(&bars->full[j % kStages], uint32_t((j / kStages) & 1), nullptr);
+        // let the copies this thread started land before the CTA can exit: the even CTA waits for its
+        // barriers (they count both CTAs' copies), the odd one gives its copies time to land
+        if (rank == 0) {
+            for (long j = issued - 1; j >= 0 && j >= issued - kStages; --j)
+                wait_phase(&bars->full[j % kStages], uint32_t((j / kStages) & 1), nullptr);
+        } else {
+            const uint64_t t0 = global_ns();
+            while (global_ns() - t0 < 100000ull) {
+            }
+        }
     }
 }
 
-template <class R>
-__device__ void mma_issuer(uint8_t* sA, uint8_t* sB, typename R::Barriers* bars, uint32_t tmem, int total,
-                           int k_iters, int32_t* flags) {
-    constexpr int kStages = R::kStages;
+// The even CTA's MMA thread.
+__device__ void mma_issuer(uint8_t* sA, uint8_t* sB, Barriers* bars, uint32_t tmem, int total, int k_iters,
+                           int32_t* flags) {
     volatile int32_t* abort = &bars->abort;
+    const int cl = int(blockIdx.x >> 1), ncl = int(gridDim.x >> 1);
     // descriptors of stage 0; a descriptor advances by (address offset) / 16
-    const uint64_t adesc0 = smem_desc<R>(smem_u32(sA)), bdesc0 = smem_desc<R>(smem_u32(sB));
+    const uint64_t adesc0 = smem_desc(smem_u32(sA)), bdesc0 = smem_desc(smem_u32(sB));
     int stage = 0;
     uint32_t phase = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
     bool ok = true;
-    for (int t = int(blockIdx.x); t < total && ok; t += int(gridDim.x)) {
+    for (int t = cl; t < total && ok; t += ncl) {
         if (!wait_phase(&bars->tempty[acc], acc_phase ^ 1u, abort)) {
             give_up(abort, flags);
             break;
@@ -248,30 +280,32 @@ __device__ void mma_issuer(uint8_t* sA, uint8_t* sB, typename R::Barriers* bars,
                 break;
             }
             tc_fence_after();
-            const uint64_t ad = adesc0 + uint64_t((stage * R::kABytes) >> 4);
-            const uint64_t bd = bdesc0 + uint64_t((stage * R::kBBytes) >> 4);
+            const uint64_t ad = adesc0 + uint64_t((stage * kABytes) >> 4);
+            const uint64_t bd = bdesc0 + uint64_t((stage * kBBytes) >> 4);
 #pragma unroll
-            for (int k16 = 0; k16 < R::kBK / 16; ++k16)  // 16 columns = 32 bytes = 2 descriptor units
-                mma_bf16(d, ad + uint64_t(2 * k16), bd + uint64_t(2 * k16), (kk | k16) != 0);
-            mma_commit(&bars->empty[stage]);
+            for (int k16 = 0; k16 < kBK / 16; ++k16)  // 16 columns = 32 bytes = 2 descriptor units
+                mma_pair(d, ad + uint64_t(2 * k16), bd + uint64_t(2 * k16), (kk | k16) != 0);
+            // release the stage to both producers: one commit for each CTA's barrier
+            mma_commit(peer_addr(&bars->empty[stage], 0));
+            mma_commit(peer_addr(&bars->empty[stage], 1));
             if (++stage == kStages) {
                 stage = 0;
                 phase ^= 1u;
             }
         }
         if (!ok) break;
-        mma_commit(&bars->tfull[acc]);
+        mma_commit(peer_addr(&bars->tfull[acc], 0));
+        mma_commit(peer_addr(&bars->tfull[acc], 1));
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1u;
     }
-    // every MMA this thread issued has finished before the CTA moves on
-    mma_commit(&bars->mma_done);
+    // every MMA this thread issued has finished before the pair moves on
+    mma_commit(peer_addr(&bars->mma_done, 0));
     wait_phase(&bars->mma_done, 0, nullptr);
 }
 
-template <class Bars>
-__device__ void epilogue(Bars* bars, uint32_t tmem, const CUtensorMap* tmC, uint8_t* sOut, int M, int N, int m_tiles,
-                         int n_tiles, int total, float4* __restrict__ partials, int32_t* flags) {
+__device__ void epilogue(Barriers* bars, uint32_t tmem, uint32_t rank, const CUtensorMap* tmC, uint8_t* sOut, int M,
+                         int N, int m_pairs, int n_tiles, int total, float4* __restrict__ partials, int32_t* flags) {
     volatile int32_t* abort = &bars->abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quarter = warp & 3;  // the TMEM lanes (rows) this warp may read
@@ -280,12 +314,14 @@ __device__ void epilogue(Bars* bars, uint32_t tmem, const CUtensorMap* tmC, uint
     // pieces permuted by the 64-byte swizzle the output tensor map applies
     const uint32_t out0 = smem_u32(sOut + (warp - 2) * 2 * kOutBlockBytes) + uint32_t(lane * 64);
     const uint32_t swz = uint32_t((lane >> 1) & 3);
+    const int cl = int(blockIdx.x >> 1), ncl = int(gridDim.x >> 1);
     int buf = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int t = int(blockIdx.x); t < total; t += int(gridDim.x)) {
-        int m, n;
-        tile_coords(t, m_tiles, n_tiles, m, n);
+    for (int t = cl; t < total; t += ncl) {
+        int mp, n;
+        tile_coords(t, m_pairs, n_tiles, mp, n);
+        const int m = 2 * mp + int(rank);
         const bool ready = wait_phase(&bars->tfull[acc], acc_phase, abort);
         if (!__all_sync(0xffffffffu, ready)) {
             give_up(abort, flags);
@@ -301,10 +337,10 @@ __device__ void epilogue(Bars* bars, uint32_t tmem, const CUtensorMap* tmC, uint
             uint32_t r[32];
             __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the per-lane branches below
             tmem_ld32(tmem + uint32_t(acc * kBN + c * 32) + lane_off, r);
-            if (c == kBN / 32 - 1) {  // the accumulator is read out: hand it back to the MMA thread
+            if (c == kBN / 32 - 1) {  // this CTA's rows are read out: tell the even CTA's MMA thread
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&bars->tempty[acc]);
+                if (lane == 0) remote_arrive(peer_addr(&bars->tempty[acc], 0));
             }
             const int col0 = n * kBN + c * 32;
             if (col0 >= N) continue;  // the same for the whole warp
@@ -342,23 +378,22 @@ __device__ void epilogue(Bars* bars, uint32_t tmem, const CUtensorMap* tmC, uint
     __syncwarp();
 }
 
-template <class R>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     lmhead_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                   const __grid_constant__ CUtensorMap tmC, int M, int N, int K, float4* __restrict__ partials,
                   int32_t* flags) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    using Barriers = typename R::Barriers;
-    constexpr int kStages = R::kStages;
     uint8_t* sB = base;
-    uint8_t* sA = base + kStages * R::kBBytes;
-    uint8_t* sOut = base + kStages * R::kStageBytes;
+    uint8_t* sA = base + kStages * kBBytes;
+    uint8_t* sOut = base + kStages * kStageBytes;
     Barriers* bars = reinterpret_cast<Barriers*>(sOut + kOutBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_rank();
     const int m_tiles = (M + kBM - 1) / kBM, n_tiles = (N + kBN - 1) / kBN;
-    const int total = m_tiles * n_tiles;
-    const int k_iters = (K + R::kBK - 1) / R::kBK;
+    const int m_pairs = (m_tiles + 1) / 2;
+    const int total = m_pairs * n_tiles;  // tiles of 256 x 256 (a pair of row tiles x one column tile)
+    const int k_iters = (K + kBK - 1) / kBK;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -367,38 +402,40 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&bars->tfull[b], 1);
-            mbar_init(&bars->tempty[b], 4);
+            mbar_init(&bars->tempty[b], 8);
         }
         mbar_init(&bars->mma_done, 1);
         bars->abort = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");  // visible to the async proxy
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmC)) : "memory");
     }
-    if (warp == 2) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&bars->tmem_base)),
+    if (warp == 2) {  // one warp of each CTA of the pair allocates, together
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&bars->tmem_base)),
                      "r"(kTmemCols)
                      : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
     }
     tc_fence_before();
     __syncthreads();
+    cluster_sync();  // both CTAs' barriers are initialised before either signals the other
     tc_fence_after();
     const uint32_t tmem = bars->tmem_base;
 
     if (warp == 0) {
-        if (lane == 0) producer<R>(&tmA, &tmB, sA, sB, bars, m_tiles, n_tiles, total, k_iters, flags);
+        if (lane == 0) producer(&tmA, &tmB, sA, sB, bars, rank, m_pairs, n_tiles, total, k_iters, flags);
     } else if (warp == 1) {
-        if (lane == 0) mma_issuer<R>(sA, sB, bars, tmem, total, k_iters, flags);
+        if (lane == 0 && rank == 0) mma_issuer(sA, sB, bars, tmem, total, k_iters, flags);
     } else {
-        epilogue(bars, tmem, &tmC, sOut, M, N, m_tiles, n_tiles, total, partials, flags);
+        epilogue(bars, tmem, rank, &tmC, sOut, M, N, m_pairs, n_tiles, total, partials, flags);
     }
     tc_fence_before();
     __syncthreads();
+    cluster_sync();  // no CTA frees its TMEM or leaves while the pair may still touch it
     if (warp == 2) {
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
     }
 }
 
@@ -464,33 +501,32 @@ bool encode_map(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Tensor maps, shared-memory opt-in and the persistent launch (one CTA per SM,
-// fewer if there are fewer tiles).  Arguments, including where the operands
-// live, are checked by the callers.
-template <class R>
+// Tensor maps, shared-memory opt-in and the persistent launch (clusters of two
+// CTAs, one CTA per SM, fewer if there are fewer tiles).  Arguments, including
+// where the operands live, are checked by the callers.
 acrl_status launch_lmhead(const acrl_bf16* hidden, int64_t M, int64_t K, int64_t ldh, const acrl_bf16* weight,
                           int64_t N, int64_t ldw, acrl_bf16* logits, int64_t ldl, float4* partials, int32_t* flags,
                           cudaStream_t s) {
     CUtensorMap tmA, tmB, tmC;
-    if (!encode_map(&tmA, hidden, uint64_t(M), uint64_t(K), uint64_t(ldh), kBM, R::kBK, R::kTmaSwizzle) ||
-        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kBN, R::kBK, R::kTmaSwizzle) ||
+    if (!encode_map(&tmA, hidden, uint64_t(M), uint64_t(K), uint64_t(ldh), kBM, kBK, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_map(&tmB, weight, uint64_t(N), uint64_t(K), uint64_t(ldw), kHalfBN, kBK, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !encode_map(&tmC, logits, uint64_t(M), uint64_t(N), uint64_t(ldl), 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
         return ACRL_ERR_CUDA;
-    if (cudaFuncSetAttribute(lmhead_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, R::kSmemBytes) !=
-        cudaSuccess)
+    if (cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess)
         return ACRL_ERR_CUDA;
-    const int64_t total = ((M + kBM - 1) / kBM) * ((N + kBN - 1) / kBN);
-    if (total > kMaxGrid) return ACRL_ERR_INVALID_ARG;
-    int dev = 0, sms = 0, per_sm = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lmhead_kernel<R>, kThreads, R::kSmemBytes) !=
-            cudaSuccess ||
-        per_sm < 1)
+    // 256 x 256 tiles; as many clusters as can be resident at once
+    const int64_t total = (((M + kBM - 1) / kBM + 1) / 2) * ((N + kBN - 1) / kBN);
+    if (total > kMaxGrid / 2) return ACRL_ERR_INVALID_ARG;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * 1024, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = s;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, lmhead_kernel, &cfg) != cudaSuccess || clusters < 1)
         return ACRL_ERR_CUDA;
-    const int64_t resident = int64_t(sms) * per_sm;
-    const int grid = int(total < resident ? total : resident);
-    lmhead_kernel<R><<<grid, kThreads, R::kSmemBytes, s>>>(tmA, tmB, tmC, int(M), int(N), int(K), partials, flags);
+    const int grid = int(2 * (total < clusters ? total : clusters));
+    lmhead_kernel<<<grid, kThreads, kSmemBytes, s>>>(tmA, tmB, tmC, int(M), int(N), int(K), partials, flags);
     return launch_status();
 }
 
@@ -538,7 +574,7 @@ extern "C" acrl_status acrl_lmhead_logits_stats(const acrl_bf16* hidden, int64_t
     if (!aligned16(hidden) || !aligned16(weight) || !aligned16(logits) || !aligned16(partials))
         return ACRL_ERR_INVALID_ARG;
     if (!operands_on_current_device({hidden, weight, logits})) return ACRL_ERR_INVALID_ARG;
-    return launch_lmhead<LmRing>(hidden, M, K, ldh, weight, N, ldw, logits, ldl, reinterpret_cast<float4*>(partials),
+    return launch_lmhead(hidden, M, K, ldh, weight, N, ldw, logits, ldl, reinterpret_cast<float4*>(partials),
                                  dev_flags, reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -610,7 +646,7 @@ extern "C" acrl_status acrl_lmhead_stats_noalloc(const acrl_bf16* hidden, int64_
     float4* partials = noalloc_scratch(dev);
     if (partials == nullptr) return ACRL_ERR_CUDA;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    const acrl_status st = launch_lmhead<LmRing>(hidden, M, K, ldh, weight, N, ldw, logits, ldl, partials, dev_flags, s);
+    const acrl_status st = launch_lmhead(hidden, M, K, ldh, weight, N, ldw, logits, ldl, partials, dev_flags, s);
     if (st != ACRL_OK) return st;
     return launch_merge(partials, logits, M, N, ldl, ids, mask, lse, logp, entropy, dev_flags, s);
 }

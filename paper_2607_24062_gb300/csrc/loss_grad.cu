@@ -12,7 +12,9 @@
 // more FMA and a multiply.  Rows that carry no gradient (masked, zero
 // coefficient and no bonus, clipped) are written as zeros without reading
 // their logits.  With lse == NULL the row's log-sum-exp is first recomputed
-// by a sweep over the same row.
+// by a sweep over the same row; the first kKeepVecs 16-byte vectors of the row
+// (96 KB) stay in the CTA's shared memory between the two sweeps, so that only
+// the rest of the row is read again, from L2.
 #include "acrl_device.cuh"
 #include "acrl_host.h"
 #include "row_lse.cuh"
@@ -21,6 +23,14 @@ namespace acrl {
 namespace {
 
 constexpr uint32_t kSignPair = 0x80008000u;
+
+// Recompute path of the CTA kernel: vectors of a row kept in shared memory
+// between the sweeps (96 KB; two 512-thread CTAs per SM), a multiple of the
+// sweep's chunk (threads x unroll vectors) so that the folds are grouped as
+// in a sweep without it.
+constexpr int kCtaThreads = 512, kCtaUnroll = 4;
+constexpr int kKeepVecs = 3 * kCtaThreads * kCtaUnroll;
+static_assert(kKeepVecs * 16 <= 100 * 1024, "two CTAs per SM must fit");
 
 // Per-row constants of the streaming pass.
 struct RowPlan {
@@ -74,21 +84,66 @@ __device__ __forceinline__ uint4 grad_vec(const uint4 v, const RowPlan& rp, int 
     return o;
 }
 
-// LAST: this is the second sweep over a row whose lines the first sweep kept in
-// L2, and the last read of them (L2 evict-first policy).  It runs backwards,
-// so that it starts on the lines the first sweep loaded last, the ones most
-// likely still in L2.
+// First sweep of the recompute path: the thread's partial state over its share
+// of the row.  Its vectors below `s` are read once from HBM (L2 evict-first:
+// they are not read from L2 again) and copied to `keep` (shared memory,
+// indexed by vector); the rest are loaded with the L2 evict-last policy,
+// since the second sweep reads them again.
+template <int TEAM, int UNROLL>
+__device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict__ row, int V, int tid, float& mx,
+                                                    uint4* __restrict__ keep, int s) {
+    LseAcc acc = lse_empty();
+    mx = -INFINITY;
+    const int nvec = V >> 3;
+    const uint4* vrow = reinterpret_cast<const uint4*>(row);
+    const uint64_t pol = policy_evict_last(), once = policy_evict_first();
+    int v = tid;
+    for (; v + (UNROLL - 1) * TEAM < s; v += UNROLL * TEAM) {
+        uint4 buf[UNROLL];
+#pragma unroll
+        for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(vrow + v + k * TEAM, once);
+#pragma unroll
+        for (int k = 0; k < UNROLL; ++k) keep[v + k * TEAM] = buf[k];
+        fold_vectors<UNROLL>(acc, mx, buf);
+    }
+    for (; v < s; v += TEAM) {
+        uint4 buf[1] = {ld_policy(vrow + v, once)};
+        keep[v] = buf[0];
+        fold_vectors<1>(acc, mx, buf);
+    }
+    for (; v + (UNROLL - 1) * TEAM < nvec; v += UNROLL * TEAM) {
+        uint4 buf[UNROLL];
+#pragma unroll
+        for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(vrow + v + k * TEAM, pol);
+        fold_vectors<UNROLL>(acc, mx, buf);
+    }
+    for (; v < nvec; v += TEAM) {
+        uint4 buf[1] = {ld_policy(vrow + v, pol)};
+        fold_vectors<1>(acc, mx, buf);
+    }
+    for (int j = (nvec << 3) + tid; j < V; j += TEAM) fold_scalar(acc, mx, bf16_to_float(row[j]));
+    return acc;
+}
+
+// LAST: this is the second sweep over a row after recompute_partial, and the
+// last read of its lines (L2 evict-first policy).  It runs backwards, so that
+// it starts on the lines the first sweep loaded last, the ones most likely
+// still in L2, and ends on the vectors below `s`, which it reads from `keep`.
 template <int TEAM, int UNROLL, bool ENT, bool LAST = false>
 __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ row, acrl_bf16* __restrict__ grow, int V,
-                                                int tid, const RowPlan& rp) {
+                                                int tid, const RowPlan& rp, const uint4* __restrict__ keep = nullptr,
+                                                int s = 0) {
     const int nvec = V >> 3;
     const uint4* src = reinterpret_cast<const uint4*>(row);
     uint4* dst = reinterpret_cast<uint4*>(grow);
     if (LAST) {
         const uint64_t pol = policy_evict_first();
-        // this thread's vectors are tid + i TEAM for i < mine; visit i = mine-1 down to 0
-        int i = tid < nvec ? (nvec - 1 - tid) / TEAM + 1 : 0;
-        for (; i >= UNROLL; i -= UNROLL) {
+        // this thread's vectors are tid + i TEAM for i < mine, those with i < i_keep in `keep`;
+        // visit i = mine-1 down to 0
+        const int mine = tid < nvec ? (nvec - 1 - tid) / TEAM + 1 : 0;
+        const int i_keep = tid < s ? min(mine, (s - 1 - tid) / TEAM + 1) : 0;
+        int i = mine;
+        for (; i - UNROLL >= i_keep; i -= UNROLL) {
             uint4 buf[UNROLL];
 #pragma unroll
             for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(src + tid + (i - 1 - k) * TEAM, pol);
@@ -98,9 +153,13 @@ __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ ro
                 st_stream(dst + vi, grad_vec<ENT>(buf[k], rp, rp.a - (vi << 3)));
             }
         }
-        for (; i > 0; --i) {
+        for (; i > i_keep; --i) {
             const int vi = tid + (i - 1) * TEAM;
             st_stream(dst + vi, grad_vec<ENT>(ld_policy(src + vi, pol), rp, rp.a - (vi << 3)));
+        }
+        for (; i > 0; --i) {
+            const int vi = tid + (i - 1) * TEAM;
+            st_stream(dst + vi, grad_vec<ENT>(keep[vi], rp, rp.a - (vi << 3)));
         }
     } else {
         int v = tid;
@@ -182,7 +241,10 @@ __device__ __forceinline__ void lse_logp(const LseAcc& acc, float mx, float za, 
 }
 
 // One row handled by a team (a whole CTA, or one warp).  `part`/`part_mx` are
-// the CTA's shared scratch for the recompute sweep (unused by warp teams).
+// the CTA's shared scratch for the recompute sweep, two buffers of one slot
+// per warp used in turn (`par`, flipped at every row that uses them; unused by
+// warp teams); `keep` holds the row's first `keep_vecs` vectors between the
+// two sweeps of the recompute path (none for warp teams).
 template <int TEAM, int UNROLL, bool RECOMPUTE, bool ENT>
 __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, int64_t t, int V, int64_t ld,
                                          const int32_t* __restrict__ ids, const uint8_t* __restrict__ mask,
@@ -190,7 +252,7 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
                                          const float* __restrict__ coef, const float* __restrict__ entropy,
                                          const float* __restrict__ ent_coef, float eps, acrl_bf16* __restrict__ grad,
                                          float* __restrict__ token_loss, int32_t* flags, int tid, LseAcc* part,
-                                         float* part_mx) {
+                                         float* part_mx, int& par, uint4* keep, int keep_vecs) {
     const acrl_bf16* row = logits + t * ld;
     acrl_bf16* grow = grad + t * ld;
     const bool m = mask ? mask[t] != 0 : true;
@@ -205,23 +267,33 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
         za = bf16_to_float(row[a]);
         if (RECOMPUTE) {
             float mx;
-            LseAcc acc = warp_lse(row_partial<TEAM, UNROLL, true>(row, V, tid, mx));
+            LseAcc acc = warp_lse(recompute_partial<TEAM, UNROLL>(row, V, tid, mx, keep, keep_vecs));
             mx = warp_max(mx);
             if (TEAM > 32) {
+                // Every warp combines the warps' states with the same butterfly, so all threads hold the same
+                // result with one barrier.  The next write to this buffer comes two rows later, after the next
+                // row's barrier, which every warp reaches only once it has read this one.
                 constexpr int NW = TEAM / 32;
-                if ((tid & 31) == 0) {
-                    part[tid >> 5] = acc;
-                    part_mx[tid >> 5] = mx;
+                static_assert(NW <= 32 && (NW & (NW - 1)) == 0, "warps per team");
+                const int lane = tid & 31;
+                LseAcc* pp = part + par * NW;
+                float* pm = part_mx + par * NW;
+                if (lane == 0) {
+                    pp[tid >> 5] = acc;
+                    pm[tid >> 5] = mx;
                 }
                 __syncthreads();
-                acc = part[0];
-                mx = part_mx[0];
+                acc = lane < NW ? pp[lane] : lse_empty();
+                mx = lane < NW ? pm[lane] : -INFINITY;
 #pragma unroll
-                for (int w = 1; w < NW; ++w) {
-                    acc = lse_merge(acc, part[w]);
-                    mx = fmaxf(mx, part_mx[w]);
+                for (int o = NW / 2; o >= 1; o >>= 1) {
+                    acc = lse_merge(acc, shfl_xor(acc, o));
+                    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
                 }
-                __syncthreads();
+                acc = LseAcc{__shfl_sync(0xffffffffu, acc.U, 0), __shfl_sync(0xffffffffu, acc.s0, 0),
+                             __shfl_sync(0xffffffffu, acc.s1, 0)};
+                mx = __shfl_sync(0xffffffffu, mx, 0);
+                par ^= 1;
             }
             lse_logp(acc, mx, za, L, lp);
         } else {
@@ -240,7 +312,8 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
     if (c == 0.f && e == 0.f) {
         zero_row<TEAM>(grow, V, tid);
     } else {
-        stream_grad_row<TEAM, UNROLL, ENT, RECOMPUTE>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a));
+        stream_grad_row<TEAM, UNROLL, ENT, RECOMPUTE>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a), keep,
+                                                      keep_vecs);
     }
 }
 
@@ -250,11 +323,15 @@ __global__ void __launch_bounds__(THREADS) loss_grad_cta(
     const uint8_t* __restrict__ mask, const float* __restrict__ lse, const float* __restrict__ old_logp,
     const float* __restrict__ coef, const float* __restrict__ entropy, const float* __restrict__ ent_coef, float eps,
     acrl_bf16* __restrict__ grad, float* __restrict__ token_loss, int32_t* flags) {
-    __shared__ LseAcc part[THREADS / 32];
-    __shared__ float part_mx[THREADS / 32];
+    __shared__ LseAcc part[2 * (THREADS / 32)];
+    __shared__ float part_mx[2 * (THREADS / 32)];
+    extern __shared__ uint4 keep[];  // recompute path: min(kKeepVecs, V / 8) vectors (dynamic size)
+    const int keep_vecs = RECOMPUTE ? min(kKeepVecs, V >> 3) : 0;
+    int par = 0;
     for (int64_t t = blockIdx.x; t < T; t += gridDim.x)
         grad_row<THREADS, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
-                                                  eps, grad, token_loss, flags, threadIdx.x, part, part_mx);
+                                                  eps, grad, token_loss, flags, threadIdx.x, part, part_mx, par, keep,
+                                                  keep_vecs);
 }
 
 template <int THREADS, int UNROLL, bool RECOMPUTE, bool ENT>
@@ -265,9 +342,10 @@ __global__ void __launch_bounds__(THREADS) loss_grad_warp(
     acrl_bf16* __restrict__ grad, float* __restrict__ token_loss, int32_t* flags) {
     constexpr int NW = THREADS / 32;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    int par = 0;
     for (int64_t t = int64_t(blockIdx.x) * NW + wid; t < T; t += int64_t(gridDim.x) * NW)
         grad_row<32, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps,
-                                             grad, token_loss, flags, lane, nullptr, nullptr);
+                                             grad, token_loss, flags, lane, nullptr, nullptr, par, nullptr, 0);
 }
 
 // Scalar loss: sum of token losses in a fixed order.  Each thread adds float4
@@ -300,19 +378,23 @@ __global__ void __launch_bounds__(kSumThreads) loss_sum_kernel(const float* __re
 }
 
 template <bool RECOMPUTE, bool ENT>
-void launch_loss_grad(const acrl_bf16* logits, int64_t T, int V, int64_t ld, const int32_t* ids, const uint8_t* mask,
-                      const float* lse, const float* old_logp, const float* coef, const float* entropy,
-                      const float* ent_coef, float eps, acrl_bf16* grad, float* token_loss, int32_t* flags,
-                      cudaStream_t s) {
+acrl_status launch_loss_grad(const acrl_bf16* logits, int64_t T, int V, int64_t ld, const int32_t* ids,
+                             const uint8_t* mask, const float* lse, const float* old_logp, const float* coef,
+                             const float* entropy, const float* ent_coef, float eps, acrl_bf16* grad,
+                             float* token_loss, int32_t* flags, cudaStream_t s) {
     if (V <= kWarpRowMaxV) {
         constexpr int THREADS = 256;
         loss_grad_warp<THREADS, 4, RECOMPUTE, ENT><<<unsigned(grid_for(THREADS / 32, T)), THREADS, 0, s>>>(
             logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
     } else {
-        constexpr int THREADS = 512;
-        loss_grad_cta<THREADS, 4, RECOMPUTE, ENT><<<unsigned(grid_for(1, T)), THREADS, 0, s>>>(
-            logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
+        auto kernel = loss_grad_cta<kCtaThreads, kCtaUnroll, RECOMPUTE, ENT>;
+        const int smem = RECOMPUTE ? 16 * (V >> 3 < kKeepVecs ? V >> 3 : kKeepVecs) : 0;
+        if (smem > 0 && cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+            return ACRL_ERR_CUDA;
+        kernel<<<unsigned(grid_for(1, T)), kCtaThreads, smem, s>>>(logits, T, V, ld, ids, mask, lse, old_logp, coef,
+                                                                   entropy, ent_coef, eps, grad, token_loss, flags);
     }
+    return ACRL_OK;
 }
 
 }  // namespace
@@ -335,18 +417,20 @@ extern "C" acrl_status acrl_loss_grad_logits(const acrl_bf16* logits, int64_t T,
     if (T > 0) {
         const int v = int(V);
         const bool ent = ent_coef != nullptr;
+        acrl_status st;
         if (lse && !ent)
-            launch_loss_grad<false, false>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
-                                           clip_eps, grad, token_loss, dev_flags, s);
+            st = launch_loss_grad<false, false>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
+                                                clip_eps, grad, token_loss, dev_flags, s);
         else if (lse && ent)
-            launch_loss_grad<false, true>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
-                                          clip_eps, grad, token_loss, dev_flags, s);
+            st = launch_loss_grad<false, true>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
+                                               clip_eps, grad, token_loss, dev_flags, s);
         else if (!ent)
-            launch_loss_grad<true, false>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
-                                          clip_eps, grad, token_loss, dev_flags, s);
+            st = launch_loss_grad<true, false>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
+                                               clip_eps, grad, token_loss, dev_flags, s);
         else
-            launch_loss_grad<true, true>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
-                                         clip_eps, grad, token_loss, dev_flags, s);
+            st = launch_loss_grad<true, true>(logits, T, v, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
+                                              clip_eps, grad, token_loss, dev_flags, s);
+        if (st != ACRL_OK) return st;
     }
     loss_sum_kernel<<<1, kSumThreads, 0, s>>>(token_loss, T, loss);
     return launch_status();

@@ -1,5 +1,5 @@
 // Per-row online log-sum-exp over bf16 logits, shared by the statistics
-// kernel and the gradient kernel's recompute sweep.
+// kernel, the gradient kernel's recompute sweep and the LM-head epilogue.
 #pragma once
 
 #include "acrl_device.cuh"
@@ -70,25 +70,21 @@ __device__ __forceinline__ void fold_scalar(LseAcc& acc, float& mx, float z) {
 }
 
 // The thread's partial state over its share of one row (lane `tid` of a team of TEAM threads).
-// KEEP: the row is read again soon (a second sweep), so its lines are loaded
-// with the L2 evict-last policy.
-template <int TEAM, int UNROLL, bool KEEP = false>
+template <int TEAM, int UNROLL>
 __device__ __forceinline__ LseAcc row_partial(const acrl_bf16* __restrict__ row, int V, int tid, float& mx) {
     LseAcc acc = lse_empty();
     mx = -INFINITY;
     const int nvec = V >> 3;
     const uint4* vrow = reinterpret_cast<const uint4*>(row);
-    const uint64_t pol = KEEP ? policy_evict_last() : 0;
     int v = tid;
     for (; v + (UNROLL - 1) * TEAM < nvec; v += UNROLL * TEAM) {
         uint4 buf[UNROLL];
 #pragma unroll
-        for (int k = 0; k < UNROLL; ++k)
-            buf[k] = KEEP ? ld_policy(vrow + v + k * TEAM, pol) : ld_stream(vrow + v + k * TEAM);
+        for (int k = 0; k < UNROLL; ++k) buf[k] = ld_stream(vrow + v + k * TEAM);
         fold_vectors<UNROLL>(acc, mx, buf);
     }
     for (; v < nvec; v += TEAM) {
-        uint4 buf[1] = {KEEP ? ld_policy(vrow + v, pol) : ld_stream(vrow + v)};
+        uint4 buf[1] = {ld_stream(vrow + v)};
         fold_vectors<1>(acc, mx, buf);
     }
     for (int j = (nvec << 3) + tid; j < V; j += TEAM) fold_scalar(acc, mx, bf16_to_float(row[j]));
