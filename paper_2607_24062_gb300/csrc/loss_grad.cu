@@ -126,9 +126,10 @@ __device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict_
 }
 
 // LAST: this is the second sweep over a row after recompute_partial, and the
-// last read of its lines (L2 evict-first policy).  It runs backwards, so that
-// it starts on the lines the first sweep loaded last, the ones most likely
-// still in L2, and ends on the vectors below `s`, which it reads from `keep`.
+// last read of its lines (L2 evict-first policy).  It reads the part that
+// comes from L2 in the order the first sweep loaded it, so that every line
+// waits about as long in L2 as any other, then the vectors below `s` from
+// `keep`.
 template <int TEAM, int UNROLL, bool ENT, bool LAST = false>
 __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ row, acrl_bf16* __restrict__ grow, int V,
                                                 int tid, const RowPlan& rp, const uint4* __restrict__ keep = nullptr,
@@ -138,27 +139,26 @@ __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ ro
     uint4* dst = reinterpret_cast<uint4*>(grow);
     if (LAST) {
         const uint64_t pol = policy_evict_first();
-        // this thread's vectors are tid + i TEAM for i < mine, those with i < i_keep in `keep`;
-        // visit i = mine-1 down to 0
+        // this thread's vectors are tid + i TEAM for i < mine, those with i < i_keep in `keep`
         const int mine = tid < nvec ? (nvec - 1 - tid) / TEAM + 1 : 0;
         const int i_keep = tid < s ? min(mine, (s - 1 - tid) / TEAM + 1) : 0;
-        int i = mine;
-        for (; i - UNROLL >= i_keep; i -= UNROLL) {
+        int i = i_keep;
+        for (; i + UNROLL <= mine; i += UNROLL) {
             uint4 buf[UNROLL];
 #pragma unroll
-            for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(src + tid + (i - 1 - k) * TEAM, pol);
+            for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(src + tid + (i + k) * TEAM, pol);
 #pragma unroll
             for (int k = 0; k < UNROLL; ++k) {
-                const int vi = tid + (i - 1 - k) * TEAM;
+                const int vi = tid + (i + k) * TEAM;
                 st_stream(dst + vi, grad_vec<ENT>(buf[k], rp, rp.a - (vi << 3)));
             }
         }
-        for (; i > i_keep; --i) {
-            const int vi = tid + (i - 1) * TEAM;
+        for (; i < mine; ++i) {
+            const int vi = tid + i * TEAM;
             st_stream(dst + vi, grad_vec<ENT>(ld_policy(src + vi, pol), rp, rp.a - (vi << 3)));
         }
-        for (; i > 0; --i) {
-            const int vi = tid + (i - 1) * TEAM;
+        for (i = 0; i < i_keep; ++i) {
+            const int vi = tid + i * TEAM;
             st_stream(dst + vi, grad_vec<ENT>(keep[vi], rp, rp.a - (vi << 3)));
         }
     } else {
