@@ -189,10 +189,11 @@ def test_uniform_logits_and_equal_policies():
 
 
 @pytest.mark.parametrize("beta", [0.0, 0.01])
-@pytest.mark.parametrize("V", [20011, 4099])
+@pytest.mark.parametrize("V", [20011, 4099, 151936])
 def test_old_logp_and_recomputed_lse(V, beta):
     """Cached-old path: weights from old log-probs, LSE recomputed in the gradient kernel, r != 1 with clipping
-    (CTA and warp row teams, with and without the entropy bonus)."""
+    (CTA and warp row teams; rows held whole in shared memory between the two sweeps, and rows of which the
+    first 96 KB are held there and the rest read again from L2; with and without the entropy bonus)."""
     spec = W.small_variant(W.QWEN, name="offpolicy", n_prompts=2, group_size=4, len_lo=10, len_hi=80, V=V)
     b = _gen(spec, seed=31)
     p = acrl.Params(entropy_coeff=beta)
@@ -679,13 +680,14 @@ def test_importance_weights_from_log_probs(mode):
         assert_close_rel(api.read_state(state)["X"], ostate.X, floor=1e-12, what="X")
 
 
-@pytest.mark.parametrize("V", [1, 7, 8, 9, 16383, 16384, 16385, 65535, 65536, 65537, 65544])
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 16383, 16384, 16385, 49152, 49153, 49160, 65535, 65536, 65537, 65544])
 def test_row_size_class_boundaries(V):
     """Vocabularies at the edges of the row-team size classes (one warp up to
     16,384 columns, 64 threads up to 65,536, 128 above for the statistics;
-    one warp, then 512 threads for the gradient) and of the 8-column vectors:
-    statistics and gradient against the oracle on every element, with the
-    lse recomputed in the gradient kernel as well."""
+    one warp, then 512 threads for the gradient), of the 8-column vectors and
+    of the part of a row the recompute path holds in shared memory (49,152
+    columns): statistics and gradient against the oracle on every element,
+    with the lse recomputed in the gradient kernel as well."""
     T = 37
     ld = ((V + 7) // 8) * 8
     gen = torch.Generator(device=DEV).manual_seed(V)
