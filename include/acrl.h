@@ -329,7 +329,11 @@ acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params
  * (H_t = -sum_j p_tj log p_tj; d H / d z_j = -p_j (log p_j + H)).
  * The probabilities are never stored.  Rows with m_t = 0, or with no
  * gradient (coef_t g_t = 0 and no entropy bonus), get a zero gradient row
- * without reading the rest of their logits.
+ * without reading the rest of their logits.  A row that carries a gradient
+ * but whose lse (given or recomputed) or log-prob is not finite (a NaN or an
+ * infinity among its logits), or whose old_logp is NaN, has no defined
+ * surrogate: its gradient row and token_loss_t are NaN (and so is *loss), and
+ * the call raises ACRL_FLAG_NONFINITE.
  *   logits  device bf16 [T, ld];  grad  device bf16 [T, ld] output (columns
  *           >= V untouched).  May be called on a chunk of rows: every
  *           per-token pointer then points at the chunk's first row.

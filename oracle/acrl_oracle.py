@@ -34,7 +34,9 @@ readings of the CUDA path; each is listed with its reason in the design notes):
     row is 0.  A row whose coefficient is 0 has a zero gradient row.
   * Any non-finite logit in a valid row makes that row's lse/logp/entropy NaN
     and sets a flag; a sampled id outside [0, V) gives logp = 0, a zero
-    gradient row and a flag.
+    gradient row and a flag.  In the gradient, a live row whose log-sum-exp
+    or log-prob is not finite, or whose old log-prob is NaN, gets a NaN token
+    loss and a NaN gradient row (and the call sets the flag).
   * A log-ratio of +inf (mu = 0 on the sampled token) follows min(rho^alpha, C)
     with rho^0 = 1; a NaN log-ratio gets weight 0 and sets a flag.
 
@@ -469,26 +471,40 @@ def loss_grad_logits(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq,
             token_loss[t] = 0.0
             total.append(0.0)
             continue
-        row = z[k]
-        if lse is None:
-            top = row.max()
-            lse_t = top + np.log(np.sum(np.exp(row - top)))
-        else:
-            lse_t = float(lse[t])
-        logp_t = row[a] - lse_t
-        r = 1.0 if old_logp is None else math.exp(logp_t - float(old_logp[t]))
         g_idx = int(seq["group"][i])
         if params.agg == AGG_TOKEN_MEAN:
             norm = float(batch["n_tokens"])
         else:
             norm = float(batch["n_groups_valid"]) * float(grp["n_valid_seqs"][g_idx]) * float(seq["n"][i])
         Ai = A[i]
+        beta = params.entropy_coeff / norm
+        if w[t] * Ai == 0.0 and beta == 0.0:
+            # reading c18: a row whose weighted advantage is 0 contributes nothing; its logits are not needed
+            token_loss[t] = 0.0
+            total.append(0.0)
+            continue
+        row = z[k]
+        with np.errstate(invalid="ignore"):     # a non-finite row gives a non-finite lse, handled below
+            if lse is None:
+                top = row.max()
+                lse_t = top + np.log(np.sum(np.exp(row - top)))
+            else:
+                lse_t = float(lse[t])
+            logp_t = row[a] - lse_t
+        old_t = math.nan if old_logp is None else float(old_logp[t])
+        if not (math.isfinite(lse_t) and math.isfinite(logp_t)) or (old_logp is not None and math.isnan(old_t)):
+            # reading c17: a row whose log-sum-exp or log-prob is not finite (a NaN or an infinity among its
+            # logits), or whose old log-prob is NaN, has no defined surrogate: NaN token loss and gradient row
+            token_loss[t] = math.nan
+            grad[k] = math.nan
+            total.append(math.nan)
+            continue
+        r = 1.0 if old_logp is None else math.exp(logp_t - old_t)
         rc = min(max(r, 1.0 - eps), 1.0 + eps)
         surrogate = min(r * Ai, rc * Ai)
         token_loss[t] = -w[t] * surrogate / norm
         gate = (Ai >= 0 and r <= 1.0 + eps) or (Ai < 0 and r >= 1.0 - eps)
         coef = w[t] * (1.0 if gate else 0.0) * r * Ai / norm
-        beta = params.entropy_coeff / norm
         if coef == 0.0 and beta == 0.0:
             total.append(token_loss[t])
             continue

@@ -183,13 +183,18 @@ __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ ro
     }
 }
 
+// A gradient row of one value (`pair` holds it twice, as a bf16x2 word), written
+// without reading the logits: 0 for rows that carry no gradient, NaN for rows
+// whose surrogate is undefined.
+constexpr uint32_t kZeroPair = 0u, kNaNPair = 0x7FC07FC0u;
+
 template <int TEAM>
-__device__ __forceinline__ void zero_row(acrl_bf16* __restrict__ grow, int V, int tid) {
+__device__ __forceinline__ void fill_row(acrl_bf16* __restrict__ grow, int V, int tid, uint32_t pair) {
     const int nvec = V >> 3;
     uint4* dst = reinterpret_cast<uint4*>(grow);
-    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    const uint4 z = make_uint4(pair, pair, pair, pair);
     for (int v = tid; v < nvec; v += TEAM) st_stream(dst + v, z);
-    for (int j = (nvec << 3) + tid; j < V; j += TEAM) grow[j] = 0;
+    for (int j = (nvec << 3) + tid; j < V; j += TEAM) grow[j] = static_cast<acrl_bf16>(pair & 0xffffu);
 }
 
 struct RowCoef {
@@ -263,6 +268,7 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
     if (m && bad_id && tid == 0) raise_flag(flags, ACRL_FLAG_BAD_ID);
     const bool live = m && !bad_id && (c0 != 0.f || e != 0.f);
     float c = 0.f, loss = 0.f, L = 0.f, H = 0.f, za = 0.f, lp = 0.f;
+    bool undefined = false;
     if (live) {
         za = bf16_to_float(row[a]);
         if (RECOMPUTE) {
@@ -300,6 +306,10 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
             L = lse[t];
             lp = za - L;
         }
+        // a row whose lse or log-prob is not finite (a NaN or an infinity among its logits), or whose old
+        // log-prob is NaN, has no defined surrogate: NaN token loss and gradient row, and the flag
+        undefined = !isfinite(L) || !isfinite(lp) || (old_logp != nullptr && isnan(old_logp[t]));
+        if (undefined && tid == 0) raise_flag(flags, ACRL_FLAG_NONFINITE);
         const RowCoef rc = row_coef(c0, lp, old_logp, t, eps);
         c = rc.c;
         loss = rc.loss;
@@ -308,9 +318,11 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
             loss -= e * H;
         }
     }
-    if (tid == 0) token_loss[t] = loss;
-    if (c == 0.f && e == 0.f) {
-        zero_row<TEAM>(grow, V, tid);
+    if (tid == 0) token_loss[t] = undefined ? __int_as_float(0x7fc00000) : loss;
+    if (undefined) {
+        fill_row<TEAM>(grow, V, tid, kNaNPair);
+    } else if (c == 0.f && e == 0.f) {
+        fill_row<TEAM>(grow, V, tid, kZeroPair);
     } else {
         stream_grad_row<TEAM, UNROLL, ENT, RECOMPUTE>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a), keep,
                                                       keep_vecs);

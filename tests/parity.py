@@ -63,8 +63,8 @@ def grad_rows(grad, rows, V: int) -> np.ndarray:
 def assert_close_rel(got, ref, rel=TOL_REL, floor=0.0, what=""):
     got = np.asarray(got, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
-    bad = np.abs(got - ref) > rel * np.abs(ref) + floor
-    bad &= ~(np.isnan(got) & np.isnan(ref))
+    bad = ~(np.abs(got - ref) <= rel * np.abs(ref) + floor)   # a NaN on one side only is a mismatch
+    bad &= ~(np.isnan(got) & np.isnan(ref)) & (got != ref)    # NaN against NaN, or equal infinities, match
     if bad.any():
         k = np.flatnonzero(bad.ravel())[:5]
         raise AssertionError(f"{what}: {bad.sum()} of {bad.size} outside rel {rel} floor {floor}; "
@@ -74,8 +74,8 @@ def assert_close_rel(got, ref, rel=TOL_REL, floor=0.0, what=""):
 def assert_close_abs(got, ref, tol, what=""):
     got = np.asarray(got, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
-    bad = np.abs(got - ref) > tol
-    bad &= ~(np.isnan(got) & np.isnan(ref))
+    bad = ~(np.abs(got - ref) <= tol)   # a NaN on one side only is a mismatch
+    bad &= ~(np.isnan(got) & np.isnan(ref)) & (got != ref)    # NaN against NaN, or equal infinities, match
     if bad.any():
         k = np.flatnonzero(bad.ravel())[:5]
         raise AssertionError(f"{what}: {bad.sum()} of {bad.size} outside abs {tol}; got {got.ravel()[k]} "
@@ -97,7 +97,8 @@ def assert_grad_rows(got, ref, coef_eff, ids_rows, what="grad", row_floor=0.0):
     ok_ids = (cols >= 0) & (cols < ref.shape[1])
     r_idx = np.arange(R)[ok_ids]
     tol[r_idx, cols[ok_ids]] += 1e-5 * np.abs(np.asarray(coef_eff)[ok_ids])
-    bad = np.abs(got - ref) > tol
+    # a NaN on one side only is a mismatch; NaN against NaN, or equal infinities, match
+    bad = ~(np.abs(got - ref) <= tol) & ~(np.isnan(got) & np.isnan(ref)) & (got != ref)
     if bad.any():
         rr, cc = np.nonzero(bad)
         raise AssertionError(f"{what}: {bad.sum()} of {bad.size} elements off; first rows {rr[:5]} cols {cc[:5]} "

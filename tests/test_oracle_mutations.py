@@ -278,10 +278,21 @@ PIN_GROUPS = {
                         P.test_calibration_then_frozen, P.test_nonpositive_X_flag_and_fixed_point],
     "loss_grad_logits": [lambda: P.test_gradient_matches_autograd(False, 0.0), P.test_on_policy_loss_by_hand_and_invariants,
                          lambda: P.test_gradient_central_differences(0.0), P.test_entropy_bonus_by_hand,
-                         lambda: P.test_gradient_matches_autograd(True, 0.0), P.test_clip_gate],
+                         lambda: P.test_gradient_matches_autograd(True, 0.0), P.test_clip_gate,
+                         lambda: P.test_gradient_undefined_rows(True), lambda: P.test_gradient_undefined_rows(False)],
     "round_bf16": [P.test_round_bf16_matches_library_and_ties],
     "lmhead_logits": [P.test_lmhead_logits_small],
 }
+
+def _loss_grad_undefined_rows_zero(z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp, batch, params,
+                                   rows=None):
+    """Mistake: a row the call cannot evaluate gets a zero gradient row and token loss 0 instead of NaN."""
+    grad, tl, loss = OA._orig["loss_grad_logits"](z, ids, mask, lse, old_logp, adv, weight, seq_offsets, seq, grp,
+                                                  batch, params, rows=rows)
+    bad = np.isnan(tl)
+    tl = np.where(bad, 0.0, tl)
+    return np.where(np.isnan(grad), 0.0, grad), tl, float(np.sum(tl[~np.isnan(tl)]))
+
 
 MUTATIONS = [
     ("token_stats", "entropy sign flipped", _token_stats_entropy_sign),
@@ -317,6 +328,7 @@ MUTATIONS = [
     ("token_stats", "bad id not reported", _token_stats_no_bad_id_flag),
     ("seq_discrepancy", "bad offsets not reported", _discrepancy_no_offsets_flag),
     ("controller_step", "X <= 0 not reported", _controller_no_x_flag),
+    ("loss_grad_logits", "undefined rows given a zero gradient", _loss_grad_undefined_rows_zero),
 ]
 
 

@@ -471,6 +471,39 @@ def test_gradient_matches_autograd(with_old, beta):
     assert loss == pytest.approx(float(L.detach()), abs=1e-14)
 
 
+@pytest.mark.parametrize("recompute", [False, True])
+def test_gradient_undefined_rows(recompute):
+    """Readings c17 and c18 in the gradient.  A live row whose log-sum-exp or
+    log-prob is not finite (a NaN or an infinity among its logits), or whose
+    old log-prob is NaN, has no defined surrogate: its token loss and its whole
+    gradient row are NaN, and so is the loss.  A row with a zero weighted
+    advantage, or a masked row, stays a zero row with token loss 0 whatever
+    its logits hold.  Every other row is exactly what it is without them."""
+    rng = np.random.default_rng(41)
+    f = _fixture(rng, with_old=True)
+    p = O.Params()
+
+    def run(z, old):
+        lse = None if recompute else O.token_stats(z, f["ids"], f["mask"])[0]
+        return O.loss_grad_logits(z, f["ids"], f["mask"], lse, old, f["adv"], f["w"], f["so"], f["seq"], f["grp"],
+                                  f["batch"], p)
+
+    g0, tl0, loss0 = run(f["z"], f["old"])
+    assert np.isfinite(loss0) and np.all(np.isfinite(g0))
+    z, old = f["z"].copy(), f["old"].copy()
+    z[3, 1] = np.nan        # live (advantage -1.3)
+    z[4, 2] = np.inf        # live
+    old[9] = np.nan         # live (advantage 2.0)
+    z[6, 0] = np.nan        # advantage 0: a zero row, never read
+    z[2, :] = np.nan        # masked
+    g, tl, loss = run(z, old)
+    bad = [3, 4, 9]
+    assert np.all(np.isnan(g[bad])) and np.all(np.isnan(tl[bad])) and np.isnan(loss)
+    assert np.all(g[[2, 6]] == 0.0) and tl[2] == 0.0 and tl[6] == 0.0
+    good = [t for t in range(len(tl)) if t not in bad]
+    assert np.array_equal(g[good], g0[good]) and np.array_equal(tl[good], tl0[good])
+
+
 @pytest.mark.parametrize("beta", [0.0, 0.3])
 def test_gradient_central_differences(beta):
     rng = np.random.default_rng(33)

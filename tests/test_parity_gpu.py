@@ -236,6 +236,63 @@ def test_old_logp_and_recomputed_lse(V, beta):
         assert_loss(float(loss), oloss, otl)
 
 
+@pytest.mark.parametrize("V", [4099, 20011, 151936])
+def test_gradient_undefined_rows_on_gpu(V):
+    """Readings c17 and c18 in the gradient call: a live row with a NaN or an
+    infinite logit, or with a NaN old log-prob, gets a NaN gradient row and a
+    NaN token loss and the call raises NONFINITE, whether the lse is given
+    (from the statistics call, NaN there too) or recomputed; a row whose
+    coefficient is 0 stays a zero row with token loss 0 whatever its logits
+    hold; every other row matches the oracle element by element."""
+    spec = W.small_variant(W.QWEN, name="undefined", n_prompts=2, group_size=4, len_lo=10, len_hi=40, V=V)
+    b = _gen(spec, seed=37)
+    p = acrl.Params()
+    op = oracle_params(p)
+    h = _host_inputs(b)
+    lse0, logp0, H0 = api.token_stats(b.logits, b.ids, b.mask, V=b.V)
+    gen = torch.Generator(device=DEV).manual_seed(5)
+    old = (logp0 + 0.1 * torch.randn(b.T, generator=gen, device=DEV)).clamp(max=0.0)
+    disc = api.seq_discrepancy(old, b.logp_mu, b.mask, b.seq_offsets, b.group_offsets, H0)
+    adv = api.grpo_advantage(b.rewards, b.group_offsets, p)
+    w, coef, alpha = api.controller_step(api.controller_init(p), p, disc, b.mask, b.seq_offsets, b.group_offsets, adv)
+    torch.cuda.synchronize()
+    # the oracle's weights from the same (clean) inputs
+    z0 = rows_f64(b.logits, np.arange(b.T), b.V)
+    _, ologp0, oH0, _ = O.token_stats(z0, h["ids"], h["mask"])
+    oold_clean = host(old).astype(np.float64)
+    lr, d, seq, grp, batch, _ = O.seq_discrepancy(oold_clean, h["mu"], h["mask"], h["so"], h["go"], oH0)
+    oadv = O.grpo_advantage(h["R"], h["go"], op)
+    ow, _, _, _, _ = O.controller_step(O.controller_init(op), op, lr, h["mask"], h["so"], h["go"], seq, grp, batch,
+                                       oadv)
+    live = np.flatnonzero(host(coef) != 0)
+    assert len(live) >= 4
+    r_nan, r_inf, r_old, r_zero = (int(x) for x in live[:4])
+    coef[r_zero] = 0.0
+    ow[r_zero] = 0.0
+    logits = b.logits.clone()
+    logits[r_nan, 3] = float("nan")
+    logits[r_inf, 5] = float("inf")
+    logits[r_zero, :] = float("nan")
+    old[r_old] = float("nan")
+    z = rows_f64(logits, np.arange(b.T), b.V)
+    olse, _, _, _ = O.token_stats(z, h["ids"], h["mask"])
+    oold = host(old).astype(np.float64)
+    coef_ref = O.loss_coefficients(ow, oadv, h["mask"], h["so"], seq, grp, batch, op)
+    for recompute in (False, True):
+        flags = api.new_flags()
+        lse, _, _ = api.token_stats(logits, b.ids, b.mask, V=b.V)
+        grad, tl, loss = api.loss_grad_logits(logits, b.ids, b.mask, None if recompute else lse, old, coef,
+                                              p.clip_eps, V=b.V, flags=flags)
+        assert api.read_flags(flags) & acrl.FLAG_NONFINITE
+        ograd, otl, oloss = O.loss_grad_logits(z, h["ids"], h["mask"], None if recompute else olse, oold, oadv, ow,
+                                               h["so"], seq, grp, batch, op)
+        g = grad_rows(grad, np.arange(b.T), b.V)
+        assert np.all(np.isnan(g[[r_nan, r_inf, r_old]])) and np.all(np.isnan(host(tl)[[r_nan, r_inf, r_old]]))
+        assert np.all(g[r_zero] == 0.0) and float(host(tl)[r_zero]) == 0.0 and np.isnan(float(loss))
+        assert_grad_rows(g, ograd, np.abs(coef_ref) * 2.0 + 1e-30, h["ids"], what=f"grad (recompute {recompute})")
+        assert_close_rel(host(tl), otl, floor=1e-12, what="token_loss")
+
+
 def test_chunked_gradient_matches_whole():
     spec = W.small_variant(W.GRPO, name="chunks", n_prompts=2, group_size=4, len_lo=30, len_hi=200, V=32000)
     b = _gen(spec, seed=4)
