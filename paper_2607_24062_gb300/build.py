@@ -8,6 +8,7 @@ library with the CUDA runtime linked statically.  The ptxas resource report
 from __future__ import annotations
 
 import concurrent.futures as cf
+import fcntl
 import glob
 import os
 import shutil
@@ -59,10 +60,23 @@ def _compile(src: str) -> tuple[str, str]:
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
-    """Compile every kernel source and link libacrl.so; returns its path."""
+    """Compile every kernel source and link libacrl.so; returns its path.
+    Processes that build at the same time (the ranks of one job) take turns
+    on a lock file, and each finds the library up to date after the first."""
     if not force and up_to_date():
         return LIB
     os.makedirs(BUILD, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            if not force and up_to_date():
+                return LIB
+            return _build_locked(verbose)
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
+def _build_locked(verbose: bool) -> str:
     srcs = _sources()
     with cf.ThreadPoolExecutor(max_workers=max(1, min(len(srcs), os.cpu_count() or 1))) as ex:
         results = list(ex.map(_compile, srcs))
