@@ -13,8 +13,9 @@
 // coefficient and no bonus, clipped) are written as zeros without reading
 // their logits.  With lse == NULL the row's log-sum-exp is first recomputed
 // by a sweep over the same row; the first kKeepVecs 16-byte vectors of the row
-// (96 KB) stay in the CTA's shared memory between the two sweeps, so that only
-// the rest of the row is read again, from L2.
+// (96 KB) stay in the CTA's shared memory and the next up to kTmemVecs (128 KB)
+// in its tensor memory between the two sweeps, so that only the rest of the
+// row is read again, from L2.
 #include "acrl_device.cuh"
 #include "acrl_host.h"
 #include "row_lse.cuh"
@@ -29,8 +30,44 @@ constexpr uint32_t kSignPair = 0x80008000u;
 // sweep's chunk (threads x unroll vectors) so that the folds are grouped as
 // in a sweep without it.
 constexpr int kCtaThreads = 512, kCtaUnroll = 4;
-constexpr int kKeepVecs = 3 * kCtaThreads * kCtaUnroll;
+constexpr int kChunk = kCtaThreads * kCtaUnroll;   // vectors one sweep step of the CTA covers
+constexpr int kKeepVecs = 3 * kChunk;
 static_assert(kKeepVecs * 16 <= 100 * 1024, "two CTAs per SM must fit");
+// The next chunks of the row (whole chunks only, so that every warp takes part
+// in each tensor-memory access) go to tensor memory: each of the two CTAs on an
+// SM allocates 256 of its 512 columns, 128 lanes x 256 columns x 4 bytes =
+// 128 KB = 4 chunks.  Thread t of warp w keeps its k-th vector of chunk c in
+// lane 32 (w mod 4) + t, columns 64 (w / 4) + 16 c + 4 k .. + 3.
+constexpr uint32_t kTmemCols = 256;
+constexpr int kTmemChunks = 4;
+constexpr int kTmemVecs = kTmemChunks * kChunk;
+static_assert(kTmemVecs * 16 == 128 * kTmemCols * 4, "tensor-memory share of a CTA");
+static_assert(kCtaThreads == 512 && kCtaUnroll == 4, "column layout: 16 warps, 4 vectors per step");
+
+// Where the vectors of a row live between the two sweeps of the recompute
+// path: [0, s) in `smem`, [s, s + tm_chunks kChunk) in tensor memory from the
+// thread's column base `tbase`, the rest in L2.
+struct RowKeep {
+    uint4* smem;
+    int s;
+    uint32_t tbase;
+    int tm_chunks;
+};
+
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint4& v) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+__device__ __forceinline__ uint4 tmem_ld4(uint32_t taddr) {
+    uint4 v;
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(taddr));
+    return v;
+}
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
 // Per-row constants of the streaming pass.
 struct RowPlan {
@@ -85,31 +122,43 @@ __device__ __forceinline__ uint4 grad_vec(const uint4 v, const RowPlan& rp, int 
 }
 
 // First sweep of the recompute path: the thread's partial state over its share
-// of the row.  Its vectors below `s` are read once from HBM (L2 evict-first:
-// they are not read from L2 again) and copied to `keep` (shared memory,
-// indexed by vector); the rest are loaded with the L2 evict-last policy,
-// since the second sweep reads them again.
+// of the row.  Its vectors below `kp.s` (read once from HBM, L2 evict-first:
+// they are not read from L2 again) are copied to shared memory (indexed by
+// vector), those of the next kp.tm_chunks whole chunks to tensor memory; the
+// rest are loaded with the L2 evict-last policy, since the second sweep reads
+// them again.  The tensor-memory stores are complete when the caller has
+// waited for them (tmem_wait_st).
 template <int TEAM, int UNROLL>
 __device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict__ row, int V, int tid, float& mx,
-                                                    uint4* __restrict__ keep, int s) {
+                                                    const RowKeep& kp) {
     LseAcc acc = lse_empty();
     mx = -INFINITY;
     const int nvec = V >> 3;
     const uint4* vrow = reinterpret_cast<const uint4*>(row);
     const uint64_t pol = policy_evict_last(), once = policy_evict_first();
+    const int s = kp.s;
     int v = tid;
     for (; v + (UNROLL - 1) * TEAM < s; v += UNROLL * TEAM) {
         uint4 buf[UNROLL];
 #pragma unroll
         for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(vrow + v + k * TEAM, once);
 #pragma unroll
-        for (int k = 0; k < UNROLL; ++k) keep[v + k * TEAM] = buf[k];
+        for (int k = 0; k < UNROLL; ++k) kp.smem[v + k * TEAM] = buf[k];
         fold_vectors<UNROLL>(acc, mx, buf);
     }
     for (; v < s; v += TEAM) {
         uint4 buf[1] = {ld_policy(vrow + v, once)};
-        keep[v] = buf[0];
+        kp.smem[v] = buf[0];
         fold_vectors<1>(acc, mx, buf);
+    }
+    // whole chunks (s is a multiple of the chunk whenever kp.tm_chunks > 0): every thread takes part
+    for (int ch = 0; ch < kp.tm_chunks; ++ch, v += UNROLL * TEAM) {
+        uint4 buf[UNROLL];
+#pragma unroll
+        for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(vrow + v + k * TEAM, once);
+#pragma unroll
+        for (int k = 0; k < UNROLL; ++k) tmem_st4(kp.tbase + uint32_t(16 * ch + 4 * k), buf[k]);
+        fold_vectors<UNROLL>(acc, mx, buf);
     }
     for (; v + (UNROLL - 1) * TEAM < nvec; v += UNROLL * TEAM) {
         uint4 buf[UNROLL];
@@ -128,39 +177,42 @@ __device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict_
 // LAST: this is the second sweep over a row after recompute_partial, and the
 // last read of its lines (L2 evict-first policy).  It reads the part that
 // comes from L2 in the order the first sweep loaded it, so that every line
-// waits about as long in L2 as any other, then the vectors below `s` from
-// `keep`.
+// waits about as long in L2 as any other, then the chunks in tensor memory,
+// then the vectors in shared memory.
 template <int TEAM, int UNROLL, bool ENT, bool LAST = false>
 __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ row, acrl_bf16* __restrict__ grow, int V,
-                                                int tid, const RowPlan& rp, const uint4* __restrict__ keep = nullptr,
-                                                int s = 0) {
+                                                int tid, const RowPlan& rp, const RowKeep& kp = RowKeep{nullptr, 0, 0u, 0}) {
     const int nvec = V >> 3;
     const uint4* src = reinterpret_cast<const uint4*>(row);
     uint4* dst = reinterpret_cast<uint4*>(grow);
     if (LAST) {
         const uint64_t pol = policy_evict_first();
-        // this thread's vectors are tid + i TEAM for i < mine, those with i < i_keep in `keep`
-        const int mine = tid < nvec ? (nvec - 1 - tid) / TEAM + 1 : 0;
-        const int i_keep = tid < s ? min(mine, (s - 1 - tid) / TEAM + 1) : 0;
-        int i = i_keep;
-        for (; i + UNROLL <= mine; i += UNROLL) {
+        const int te = kp.s + kp.tm_chunks * UNROLL * TEAM;   // first vector read from L2
+        int v = te + tid;
+        for (; v + (UNROLL - 1) * TEAM < nvec; v += UNROLL * TEAM) {
             uint4 buf[UNROLL];
 #pragma unroll
-            for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(src + tid + (i + k) * TEAM, pol);
+            for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(src + v + k * TEAM, pol);
 #pragma unroll
             for (int k = 0; k < UNROLL; ++k) {
-                const int vi = tid + (i + k) * TEAM;
+                const int vi = v + k * TEAM;
                 st_stream(dst + vi, grad_vec<ENT>(buf[k], rp, rp.a - (vi << 3)));
             }
         }
-        for (; i < mine; ++i) {
-            const int vi = tid + i * TEAM;
-            st_stream(dst + vi, grad_vec<ENT>(ld_policy(src + vi, pol), rp, rp.a - (vi << 3)));
+        for (; v < nvec; v += TEAM) st_stream(dst + v, grad_vec<ENT>(ld_policy(src + v, pol), rp, rp.a - (v << 3)));
+        for (int ch = 0; ch < kp.tm_chunks; ++ch) {
+            uint4 buf[UNROLL];
+#pragma unroll
+            for (int k = 0; k < UNROLL; ++k) buf[k] = tmem_ld4(kp.tbase + uint32_t(16 * ch + 4 * k));
+            tmem_wait_ld();
+            const int v0 = kp.s + ch * UNROLL * TEAM + tid;
+#pragma unroll
+            for (int k = 0; k < UNROLL; ++k) {
+                const int vi = v0 + k * TEAM;
+                st_stream(dst + vi, grad_vec<ENT>(buf[k], rp, rp.a - (vi << 3)));
+            }
         }
-        for (i = 0; i < i_keep; ++i) {
-            const int vi = tid + i * TEAM;
-            st_stream(dst + vi, grad_vec<ENT>(keep[vi], rp, rp.a - (vi << 3)));
-        }
+        for (int vi = tid; vi < kp.s; vi += TEAM) st_stream(dst + vi, grad_vec<ENT>(kp.smem[vi], rp, rp.a - (vi << 3)));
     } else {
         int v = tid;
         for (; v + (UNROLL - 1) * TEAM < nvec; v += UNROLL * TEAM) {
@@ -248,8 +300,8 @@ __device__ __forceinline__ void lse_logp(const LseAcc& acc, float mx, float za, 
 // One row handled by a team (a whole CTA, or one warp).  `part`/`part_mx` are
 // the CTA's shared scratch for the recompute sweep, two buffers of one slot
 // per warp used in turn (`par`, flipped at every row that uses them; unused by
-// warp teams); `keep` holds the row's first `keep_vecs` vectors between the
-// two sweeps of the recompute path (none for warp teams).
+// warp teams); `kp` says where the recompute path keeps the row between its
+// two sweeps (nothing on chip for warp teams).
 template <int TEAM, int UNROLL, bool RECOMPUTE, bool ENT>
 __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, int64_t t, int V, int64_t ld,
                                          const int32_t* __restrict__ ids, const uint8_t* __restrict__ mask,
@@ -257,7 +309,7 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
                                          const float* __restrict__ coef, const float* __restrict__ entropy,
                                          const float* __restrict__ ent_coef, float eps, acrl_bf16* __restrict__ grad,
                                          float* __restrict__ token_loss, int32_t* flags, int tid, LseAcc* part,
-                                         float* part_mx, int& par, uint4* keep, int keep_vecs) {
+                                         float* part_mx, int& par, const RowKeep& kp) {
     const acrl_bf16* row = logits + t * ld;
     acrl_bf16* grow = grad + t * ld;
     const bool m = mask ? mask[t] != 0 : true;
@@ -273,7 +325,8 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
         za = bf16_to_float(row[a]);
         if (RECOMPUTE) {
             float mx;
-            LseAcc acc = warp_lse(recompute_partial<TEAM, UNROLL>(row, V, tid, mx, keep, keep_vecs));
+            LseAcc acc = warp_lse(recompute_partial<TEAM, UNROLL>(row, V, tid, mx, kp));
+            if (kp.tm_chunks > 0) tmem_wait_st();   // before the barrier: the row's tensor-memory part is written
             mx = warp_max(mx);
             if (TEAM > 32) {
                 // Every warp combines the warps' states with the same butterfly, so all threads hold the same
@@ -324,8 +377,7 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
     } else if (c == 0.f && e == 0.f) {
         fill_row<TEAM>(grow, V, tid, kZeroPair);
     } else {
-        stream_grad_row<TEAM, UNROLL, ENT, RECOMPUTE>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a), keep,
-                                                      keep_vecs);
+        stream_grad_row<TEAM, UNROLL, ENT, RECOMPUTE>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a), kp);
     }
 }
 
@@ -337,13 +389,42 @@ __global__ void __launch_bounds__(THREADS) loss_grad_cta(
     acrl_bf16* __restrict__ grad, float* __restrict__ token_loss, int32_t* flags) {
     __shared__ LseAcc part[2 * (THREADS / 32)];
     __shared__ float part_mx[2 * (THREADS / 32)];
+    __shared__ uint32_t tmem_base;
     extern __shared__ uint4 keep[];  // recompute path: min(kKeepVecs, V / 8) vectors (dynamic size)
-    const int keep_vecs = RECOMPUTE ? min(kKeepVecs, V >> 3) : 0;
+    const int warp = threadIdx.x >> 5;
+    RowKeep kp{keep, 0, 0u, 0};
+    if (RECOMPUTE) {
+        static_assert(!RECOMPUTE || (THREADS == kCtaThreads && UNROLL == kCtaUnroll), "tensor-memory layout");
+        const int nvec = V >> 3;
+        kp.s = min(kKeepVecs, nvec);
+        kp.tm_chunks = nvec > kKeepVecs ? min(kTmemChunks, (nvec - kKeepVecs) / kChunk) : 0;
+        if (kp.tm_chunks > 0) {   // the same for every CTA of the launch
+            if (warp == 0) {
+                asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                                 static_cast<uint32_t>(__cvta_generic_to_shared(&tmem_base))),
+                             "r"(kTmemCols)
+                             : "memory");
+                asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncthreads();
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            kp.tbase = tmem_base + (uint32_t((warp & 3) * 32) << 16) + uint32_t((warp >> 2) * 64);
+        }
+    }
     int par = 0;
     for (int64_t t = blockIdx.x; t < T; t += gridDim.x)
         grad_row<THREADS, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
-                                                  eps, grad, token_loss, flags, threadIdx.x, part, part_mx, par, keep,
-                                                  keep_vecs);
+                                                  eps, grad, token_loss, flags, threadIdx.x, part, part_mx, par, kp);
+    if (RECOMPUTE && kp.tm_chunks > 0) {   // every tensor-memory read has completed (tmem_wait_ld)
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        if (warp == 0) {
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(kTmemCols)
+                         : "memory");
+        }
+    }
 }
 
 template <int THREADS, int UNROLL, bool RECOMPUTE, bool ENT>
@@ -357,7 +438,8 @@ __global__ void __launch_bounds__(THREADS) loss_grad_warp(
     int par = 0;
     for (int64_t t = int64_t(blockIdx.x) * NW + wid; t < T; t += int64_t(gridDim.x) * NW)
         grad_row<32, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps,
-                                             grad, token_loss, flags, lane, nullptr, nullptr, par, nullptr, 0);
+                                             grad, token_loss, flags, lane, nullptr, nullptr, par,
+                                             RowKeep{nullptr, 0, 0u, 0});
 }
 
 // Scalar loss: sum of token losses in a fixed order.  Each thread adds float4
