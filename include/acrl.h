@@ -71,8 +71,10 @@ typedef enum {
 #define ACRL_FLAG_NONFINITE   0x2   /* a valid row held a NaN or an infinity   */
 #define ACRL_FLAG_BAD_OFFSETS 0x4   /* seq/group offsets not monotone or not covering */
 #define ACRL_FLAG_X_NONPOS    0x8   /* ACRL mode with a reference X <= 0       */
-#define ACRL_FLAG_TIMEOUT     0x10  /* a pipeline wait inside the tensor-core kernel gave
-                                       up after its time limit: that call's outputs are invalid */
+#define ACRL_FLAG_TIMEOUT     0x10  /* a bounded wait inside a kernel (the tensor-core
+                                       pipeline, or the bulk copy of the lse-recompute
+                                       gradient) gave up after its time limit: that call's
+                                       outputs are invalid */
 
 /* Importance-weight mode. */
 typedef enum {
@@ -341,9 +343,11 @@ acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params
  *   lse     device float [T] from acrl_token_stats on the same logits, or
  *           NULL to recompute it here (the cached-old path: a second sweep
  *           over each row; for rows of more than 16,384 columns each CTA
- *           keeps up to 96 KB of its row in shared memory and, above 49,152
- *           columns, up to 128 KB in tensor memory between the sweeps: it
- *           allocates 256 of the SM's 512 tensor-memory columns while it runs).
+ *           keeps up to 96 KB of its row in shared memory, loaded by one
+ *           bulk copy per row whose wait is bounded (ACRL_FLAG_TIMEOUT), and,
+ *           above 49,152 columns, up to 128 KB in tensor memory between the
+ *           sweeps: it allocates 256 of the SM's 512 tensor-memory columns
+ *           while it runs).
  *   old_logp  device float [T] log pi_old(a_t), or NULL for r = 1.
  *   coef    device float [T]: acrl_controller_step's `coef` output for the
  *           same batch (the same rows, in the same order).  It carries

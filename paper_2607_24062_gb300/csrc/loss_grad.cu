@@ -15,9 +15,11 @@
 // by a sweep over the same row; the first kKeepVecs 16-byte vectors of the row
 // (96 KB) stay in the CTA's shared memory and the next up to kTmemVecs (128 KB)
 // in its tensor memory between the two sweeps, so that only the rest of the
-// row is read again, from L2.
+// row is read again, from L2.  The shared-memory part arrives by one bulk copy
+// started when the row starts, while the threads load the rest.
 #include "acrl_device.cuh"
 #include "acrl_host.h"
+#include "mbarrier.cuh"
 #include "row_lse.cuh"
 
 namespace acrl {
@@ -51,14 +53,26 @@ static_assert(kTmemVecs * 16 == 128 * kTmemCols * 4, "tensor-memory share of a C
 static_assert(kCtaThreads == 512 && kCtaUnroll == 4, "column layout: 16 warps, 4 vectors per step");
 
 // Where the vectors of a row live between the two sweeps of the recompute
-// path: [0, s) in `smem`, [s, s + tm_chunks kChunk) in tensor memory from the
-// thread's column base `tbase`, the rest in L2.
+// path: [0, s) in `smem` (filled by a bulk copy that completes on `bar`),
+// [s, s + tm_chunks kChunk) in tensor memory from the thread's column base
+// `tbase`, the rest in L2.
 struct RowKeep {
     uint4* smem;
     int s;
     uint32_t tbase;
     int tm_chunks;
+    uint64_t* bar;
 };
+
+// Bulk copy of `bytes` (a multiple of 16; both addresses 16-byte aligned) from
+// global to this CTA's shared memory, completing on `bar`, with an L2 policy.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::
+            "r"(smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(pol)
+        : "memory");
+}
 
 __device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint4& v) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(v.x), "r"(v.y),
@@ -128,35 +142,24 @@ __device__ __forceinline__ uint4 grad_vec(const uint4 v, const RowPlan& rp, int 
 }
 
 // First sweep of the recompute path: the thread's partial state over its share
-// of the row.  Its vectors below `kp.s` (read once from HBM, L2 evict-first:
-// they are not read from L2 again) are copied to shared memory (indexed by
-// vector), those of the next kp.tm_chunks whole chunks to tensor memory; the
-// rest are loaded with the L2 evict-last policy, since the second sweep reads
-// them again.  The tensor-memory stores are complete when the caller has
-// waited for them (tmem_wait_st).
+// of the row.  Vectors below `kp.s` (read once from HBM, L2 evict-first: they
+// are not read from L2 again) come into shared memory by the bulk copy that
+// thread 0 started on `kp.bar` (phase parity `parity`) and are folded last,
+// once it has landed; those of the next kp.tm_chunks whole chunks are copied
+// to tensor memory; the rest are loaded with the L2 evict-last policy, since
+// the second sweep reads them again.  The tensor-memory stores are complete
+// when the caller has waited for them (tmem_wait_st).  A copy that has not
+// landed after the bounded wait raises ACRL_FLAG_TIMEOUT.
 template <int TEAM, int UNROLL>
 __device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict__ row, int V, int tid, float& mx,
-                                                    const RowKeep& kp) {
+                                                    const RowKeep& kp, uint32_t parity, int32_t* flags) {
     LseAcc acc = lse_empty();
     mx = -INFINITY;
     const int nvec = V >> 3;
     const uint4* vrow = reinterpret_cast<const uint4*>(row);
     const uint64_t pol = policy_evict_last(), once = policy_evict_first();
     const int s = kp.s;
-    int v = tid;
-    for (; v + (UNROLL - 1) * TEAM < s; v += UNROLL * TEAM) {
-        uint4 buf[UNROLL];
-#pragma unroll
-        for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(vrow + v + k * TEAM, once);
-#pragma unroll
-        for (int k = 0; k < UNROLL; ++k) kp.smem[v + k * TEAM] = buf[k];
-        fold_vectors<UNROLL>(acc, mx, buf);
-    }
-    for (; v < s; v += TEAM) {
-        uint4 buf[1] = {ld_policy(vrow + v, once)};
-        kp.smem[v] = buf[0];
-        fold_vectors<1>(acc, mx, buf);
-    }
+    int v = s + tid;
     // whole chunks (s is a multiple of the chunk whenever kp.tm_chunks > 0): every thread takes part
     for (int ch = 0; ch < kp.tm_chunks; ++ch, v += UNROLL * TEAM) {
         uint4 buf[UNROLL];
@@ -177,6 +180,19 @@ __device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict_
         fold_vectors<1>(acc, mx, buf);
     }
     for (int j = (nvec << 3) + tid; j < V; j += TEAM) fold_scalar(acc, mx, bf16_to_float(row[j]));
+    if (s > 0) {
+        if (!wait_phase(kp.bar, parity, nullptr)) raise_flag(flags, ACRL_FLAG_TIMEOUT);
+        for (v = tid; v + (UNROLL - 1) * TEAM < s; v += UNROLL * TEAM) {
+            uint4 buf[UNROLL];
+#pragma unroll
+            for (int k = 0; k < UNROLL; ++k) buf[k] = kp.smem[v + k * TEAM];
+            fold_vectors<UNROLL>(acc, mx, buf);
+        }
+        for (; v < s; v += TEAM) {
+            uint4 buf[1] = {kp.smem[v]};
+            fold_vectors<1>(acc, mx, buf);
+        }
+    }
     return acc;
 }
 
@@ -187,7 +203,8 @@ __device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict_
 // then the vectors in shared memory.
 template <int TEAM, int UNROLL, bool ENT, bool LAST = false>
 __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ row, acrl_bf16* __restrict__ grow, int V,
-                                                int tid, const RowPlan& rp, const RowKeep& kp = RowKeep{nullptr, 0, 0u, 0}) {
+                                                int tid, const RowPlan& rp,
+                                                const RowKeep& kp = RowKeep{nullptr, 0, 0u, 0, nullptr}) {
     const int nvec = V >> 3;
     const uint4* src = reinterpret_cast<const uint4*>(row);
     uint4* dst = reinterpret_cast<uint4*>(grow);
@@ -307,7 +324,10 @@ __device__ __forceinline__ void lse_logp(const LseAcc& acc, float mx, float za, 
 // the CTA's shared scratch for the recompute sweep, two buffers of one slot
 // per warp used in turn (`par`, flipped at every row that uses them; unused by
 // warp teams); `kp` says where the recompute path keeps the row between its
-// two sweeps (nothing on chip for warp teams).
+// two sweeps (nothing on chip for warp teams).  The bulk copy of the row's
+// shared-memory part is started by thread 0 once the row is known to be live,
+// and completes the phase of kp.bar whose parity is `par`: both flip at every
+// live row of a CTA team.
 template <int TEAM, int UNROLL, bool RECOMPUTE, bool ENT>
 __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, int64_t t, int V, int64_t ld,
                                          const int32_t* __restrict__ ids, const uint8_t* __restrict__ mask,
@@ -328,10 +348,16 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
     float c = 0.f, loss = 0.f, L = 0.f, H = 0.f, za = 0.f, lp = 0.f;
     bool undefined = false;
     if (live) {
+        if (RECOMPUTE && TEAM > 32 && kp.s > 0 && tid == 0) {
+            // the threads' reads of the last row's part (before the CTA barrier) come before the copy's writes
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_expect_tx(kp.bar, uint32_t(kp.s) * 16u);
+            bulk_load(kp.smem, row, uint32_t(kp.s) * 16u, kp.bar, policy_evict_first());
+        }
         za = bf16_to_float(row[a]);
         if (RECOMPUTE) {
             float mx;
-            LseAcc acc = warp_lse(recompute_partial<TEAM, UNROLL>(row, V, tid, mx, kp));
+            LseAcc acc = warp_lse(recompute_partial<TEAM, UNROLL>(row, V, tid, mx, kp, uint32_t(par), flags));
             if (kp.tm_chunks > 0) tmem_wait_st();   // before the barrier: the row's tensor-memory part is written
             mx = warp_max(mx);
             if (TEAM > 32) {
@@ -396,32 +422,39 @@ __global__ void __launch_bounds__(THREADS) loss_grad_cta(
     __shared__ LseAcc part[2 * (THREADS / 32)];
     __shared__ float part_mx[2 * (THREADS / 32)];
     __shared__ uint32_t tmem_base;
+    __shared__ __align__(8) uint64_t keep_bar;
     extern __shared__ uint4 keep[];  // recompute path: min(kKeepVecs, V / 8) vectors (dynamic size)
     const int warp = threadIdx.x >> 5;
-    RowKeep kp{keep, 0, 0u, 0};
+    RowKeep kp{keep, 0, 0u, 0, &keep_bar};
     if (RECOMPUTE) {
         static_assert(!RECOMPUTE || (THREADS == kCtaThreads && UNROLL == kCtaUnroll), "tensor-memory layout");
         const int nvec = V >> 3;
         kp.s = min(kKeepVecs, nvec);
         kp.tm_chunks = nvec > kKeepVecs ? min(kTmemChunks, (nvec - kKeepVecs) / kChunk) : 0;
-        if (kp.tm_chunks > 0) {   // the same for every CTA of the launch
-            if (warp == 0) {
-                asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                                 static_cast<uint32_t>(__cvta_generic_to_shared(&tmem_base))),
-                             "r"(kTmemCols)
-                             : "memory");
-                asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-            }
-            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-            __syncthreads();
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            kp.tbase = tmem_base + (uint32_t((warp & 3) * 32) << 16) + uint32_t((warp >> 2) * 64);
+        if (threadIdx.x == 0) {
+            mbar_init(&keep_bar, 1);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         }
+        if (kp.tm_chunks > 0 && warp == 0) {   // the same for every CTA of the launch
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             static_cast<uint32_t>(__cvta_generic_to_shared(&tmem_base))),
+                         "r"(kTmemCols)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        }
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        if (kp.tm_chunks > 0)
+            kp.tbase = tmem_base + (uint32_t((warp & 3) * 32) << 16) + uint32_t((warp >> 2) * 64);
     }
     int par = 0;
-    for (int64_t t = blockIdx.x; t < T; t += gridDim.x)
+    for (int64_t t = blockIdx.x; t < T; t += gridDim.x) {
+        // a CTA with a further row refills its shared-memory part only once every thread has read the last one
+        if (RECOMPUTE && t != blockIdx.x) __syncthreads();
         grad_row<THREADS, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
                                                   eps, grad, token_loss, flags, threadIdx.x, part, part_mx, par, kp);
+    }
     if (RECOMPUTE && kp.tm_chunks > 0) {   // every tensor-memory read has completed (tmem_wait_ld)
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         __syncthreads();
@@ -445,7 +478,7 @@ __global__ void __launch_bounds__(THREADS) loss_grad_warp(
     for (int64_t t = int64_t(blockIdx.x) * NW + wid; t < T; t += int64_t(gridDim.x) * NW)
         grad_row<32, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps,
                                              grad, token_loss, flags, lane, nullptr, nullptr, par,
-                                             RowKeep{nullptr, 0, 0u, 0});
+                                             RowKeep{nullptr, 0, 0u, 0, nullptr});
 }
 
 // Scalar loss: sum of token losses in a fixed order.  Each thread adds float4
