@@ -343,11 +343,11 @@ acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params
  *   lse     device float [T] from acrl_token_stats on the same logits, or
  *           NULL to recompute it here (the cached-old path: a second sweep
  *           over each row; for rows of more than 16,384 columns each CTA
- *           keeps up to 96 KB of its row in shared memory, loaded by one
- *           bulk copy per row whose wait is bounded (ACRL_FLAG_TIMEOUT), and,
- *           above 49,152 columns, up to 128 KB in tensor memory between the
- *           sweeps: it allocates 256 of the SM's 512 tensor-memory columns
- *           while it runs).
+ *           keeps up to 72 KB (rows of up to 40,967 columns) or 96 KB of its
+ *           row in shared memory, loaded by one bulk copy per row whose wait
+ *           is bounded (ACRL_FLAG_TIMEOUT), and, from 65,536 columns, up to
+ *           128 KB in tensor memory between the sweeps: it then allocates 256
+ *           of the SM's 512 tensor-memory columns while it runs).
  *   old_logp  device float [T] log pi_old(a_t), or NULL for r = 1.
  *   coef    device float [T]: acrl_controller_step's `coef` output for the
  *           same batch (the same rows, in the same order).  It carries

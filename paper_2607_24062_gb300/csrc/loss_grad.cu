@@ -51,6 +51,22 @@ constexpr int kTmemChunks = 4;
 constexpr int kTmemVecs = kTmemChunks * kChunk;
 static_assert(kTmemVecs * 16 == 128 * kTmemCols * 4, "tensor-memory share of a CTA");
 static_assert(kCtaThreads == 512 && kCtaUnroll == 4, "column layout: 16 warps, 4 vectors per step");
+// Tensor memory holds whole chunks only, so rows of fewer than kKeepVecs +
+// kChunk vectors (V < 65,536) keep nothing there; they take a kernel instance
+// without any tcgen05 code (TM = false).  A resident CTA of a kernel that may
+// allocate tensor memory keeps the SM from starting another CTA of that kernel
+// until it has given up its allocation permit: measured with ncu, 15.6 warps
+// resident per SM against 30.7 for the same work without tcgen05 code.
+constexpr int kTmemMinVecs = kKeepVecs + kChunk;
+// Rows of up to kSmallMaxVecs vectors (V <= 40,967) take 256-thread CTAs in
+// the recompute path, each keeping up to 72 KB of its row in shared memory so
+// that three fit on an SM (the rest of the row, at most 8 KB, is read again
+// from L2): 0.92-0.98 of the copy rate for V = 32,000-40,000 against 0.77-0.85
+// with two 512-thread CTAs per SM; from V = 44,000 the 512-thread CTAs, which
+// keep 96 KB, are ahead (0.87-0.93 against 0.82-0.87).
+constexpr int kSmallThreads = 256;
+constexpr int kSmallKeepVecs = 4608;
+constexpr int kSmallMaxVecs = 5120;
 
 // Where the vectors of a row live between the two sweeps of the recompute
 // path: [0, s) in `smem` (filled by a bulk copy that completes on `bar`),
@@ -150,7 +166,7 @@ __device__ __forceinline__ uint4 grad_vec(const uint4 v, const RowPlan& rp, int 
 // the second sweep reads them again.  The tensor-memory stores are complete
 // when the caller has waited for them (tmem_wait_st).  A copy that has not
 // landed after the bounded wait raises ACRL_FLAG_TIMEOUT.
-template <int TEAM, int UNROLL>
+template <int TEAM, int UNROLL, bool TM>
 __device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict__ row, int V, int tid, float& mx,
                                                     const RowKeep& kp, uint32_t parity, int32_t* flags) {
     LseAcc acc = lse_empty();
@@ -161,13 +177,15 @@ __device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict_
     const int s = kp.s;
     int v = s + tid;
     // whole chunks (s is a multiple of the chunk whenever kp.tm_chunks > 0): every thread takes part
-    for (int ch = 0; ch < kp.tm_chunks; ++ch, v += UNROLL * TEAM) {
-        uint4 buf[UNROLL];
+    if constexpr (TM) {
+        for (int ch = 0; ch < kp.tm_chunks; ++ch, v += UNROLL * TEAM) {
+            uint4 buf[UNROLL];
 #pragma unroll
-        for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(vrow + v + k * TEAM, once);
+            for (int k = 0; k < UNROLL; ++k) buf[k] = ld_policy(vrow + v + k * TEAM, once);
 #pragma unroll
-        for (int k = 0; k < UNROLL; ++k) tmem_st4(kp.tbase + uint32_t(16 * ch + 4 * k), buf[k]);
-        fold_vectors<UNROLL>(acc, mx, buf);
+            for (int k = 0; k < UNROLL; ++k) tmem_st4(kp.tbase + uint32_t(16 * ch + 4 * k), buf[k]);
+            fold_vectors<UNROLL>(acc, mx, buf);
+        }
     }
     for (; v + (UNROLL - 1) * TEAM < nvec; v += UNROLL * TEAM) {
         uint4 buf[UNROLL];
@@ -201,7 +219,7 @@ __device__ __forceinline__ LseAcc recompute_partial(const acrl_bf16* __restrict_
 // comes from L2 in the order the first sweep loaded it, so that every line
 // waits about as long in L2 as any other, then the chunks in tensor memory,
 // then the vectors in shared memory.
-template <int TEAM, int UNROLL, bool ENT, bool LAST = false>
+template <int TEAM, int UNROLL, bool ENT, bool LAST = false, bool TM = false>
 __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ row, acrl_bf16* __restrict__ grow, int V,
                                                 int tid, const RowPlan& rp,
                                                 const RowKeep& kp = RowKeep{nullptr, 0, 0u, 0, nullptr}) {
@@ -223,7 +241,7 @@ __device__ __forceinline__ void stream_grad_row(const acrl_bf16* __restrict__ ro
             }
         }
         for (; v < nvec; v += TEAM) st_stream(dst + v, grad_vec<ENT>(ld_policy(src + v, pol), rp, rp.a - (v << 3)));
-        for (int ch = 0; ch < kp.tm_chunks; ++ch) {
+        for (int ch = 0; TM && ch < kp.tm_chunks; ++ch) {
             uint4 buf[UNROLL];
 #pragma unroll
             for (int k = 0; k < UNROLL; ++k) buf[k] = tmem_ld4(kp.tbase + uint32_t(16 * ch + 4 * k));
@@ -328,7 +346,7 @@ __device__ __forceinline__ void lse_logp(const LseAcc& acc, float mx, float za, 
 // shared-memory part is started by thread 0 once the row is known to be live,
 // and completes the phase of kp.bar whose parity is `par`: both flip at every
 // live row of a CTA team.
-template <int TEAM, int UNROLL, bool RECOMPUTE, bool ENT>
+template <int TEAM, int UNROLL, bool RECOMPUTE, bool ENT, bool TM>
 __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, int64_t t, int V, int64_t ld,
                                          const int32_t* __restrict__ ids, const uint8_t* __restrict__ mask,
                                          const float* __restrict__ lse, const float* __restrict__ old_logp,
@@ -357,8 +375,9 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
         za = bf16_to_float(row[a]);
         if (RECOMPUTE) {
             float mx;
-            LseAcc acc = warp_lse(recompute_partial<TEAM, UNROLL>(row, V, tid, mx, kp, uint32_t(par), flags));
-            if (kp.tm_chunks > 0) tmem_wait_st();   // before the barrier: the row's tensor-memory part is written
+            LseAcc acc = warp_lse(recompute_partial<TEAM, UNROLL, TM>(row, V, tid, mx, kp, uint32_t(par), flags));
+            if (TM && kp.tm_chunks > 0)
+                tmem_wait_st();   // before the barrier: the row's tensor-memory part is written
             mx = warp_max(mx);
             if (TEAM > 32) {
                 // Every warp combines the warps' states with the same butterfly, so all threads hold the same
@@ -409,11 +428,14 @@ __device__ __forceinline__ void grad_row(const acrl_bf16* __restrict__ logits, i
     } else if (c == 0.f && e == 0.f) {
         fill_row<TEAM>(grow, V, tid, kZeroPair);
     } else {
-        stream_grad_row<TEAM, UNROLL, ENT, RECOMPUTE>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a), kp);
+        stream_grad_row<TEAM, UNROLL, ENT, RECOMPUTE, TM>(row, grow, V, tid, make_plan<ENT>(c, e, L, H, za, lp, a),
+                                                          kp);
     }
 }
 
-template <int THREADS, int UNROLL, bool RECOMPUTE, bool ENT>
+// TM: the recompute instance whose CTAs keep whole chunks of a row in tensor
+// memory (512 threads, rows of at least kTmemMinVecs vectors).
+template <int THREADS, int UNROLL, bool RECOMPUTE, bool ENT, bool TM = false>
 __global__ void __launch_bounds__(THREADS) loss_grad_cta(
     const acrl_bf16* __restrict__ logits, int64_t T, int V, int64_t ld, const int32_t* __restrict__ ids,
     const uint8_t* __restrict__ mask, const float* __restrict__ lse, const float* __restrict__ old_logp,
@@ -425,43 +447,53 @@ __global__ void __launch_bounds__(THREADS) loss_grad_cta(
     __shared__ __align__(8) uint64_t keep_bar;
     extern __shared__ uint4 keep[];  // recompute path: min(kKeepVecs, V / 8) vectors (dynamic size)
     const int warp = threadIdx.x >> 5;
+    static_assert(!TM || (RECOMPUTE && THREADS == kCtaThreads && UNROLL == kCtaUnroll), "tensor-memory layout");
     RowKeep kp{keep, 0, 0u, 0, &keep_bar};
     if (RECOMPUTE) {
-        static_assert(!RECOMPUTE || (THREADS == kCtaThreads && UNROLL == kCtaUnroll), "tensor-memory layout");
         const int nvec = V >> 3;
-        kp.s = min(kKeepVecs, nvec);
-        kp.tm_chunks = nvec > kKeepVecs ? min(kTmemChunks, (nvec - kKeepVecs) / kChunk) : 0;
+        kp.s = min(THREADS == kSmallThreads ? kSmallKeepVecs : kKeepVecs, nvec);
+        kp.tm_chunks = TM && nvec > kKeepVecs ? min(kTmemChunks, (nvec - kKeepVecs) / kChunk) : 0;
         if (threadIdx.x == 0) {
             mbar_init(&keep_bar, 1);
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         }
-        if (kp.tm_chunks > 0 && warp == 0) {   // the same for every CTA of the launch
-            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                             static_cast<uint32_t>(__cvta_generic_to_shared(&tmem_base))),
-                         "r"(kTmemCols)
-                         : "memory");
-            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        if constexpr (TM) {
+            if (warp == 0) {   // kp.tm_chunks is the same for every CTA of the launch
+                if (kp.tm_chunks > 0)
+                    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                                     static_cast<uint32_t>(__cvta_generic_to_shared(&tmem_base))),
+                                 "r"(kTmemCols)
+                                 : "memory");
+                // at once, allocation or not: the SM may then start the kernel's next CTA
+                asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         }
-        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         __syncthreads();
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        if (kp.tm_chunks > 0)
-            kp.tbase = tmem_base + (uint32_t((warp & 3) * 32) << 16) + uint32_t((warp >> 2) * 64);
+        if constexpr (TM) {
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            if (kp.tm_chunks > 0)
+                kp.tbase = tmem_base + (uint32_t((warp & 3) * 32) << 16) + uint32_t((warp >> 2) * 64);
+        }
     }
     int par = 0;
     for (int64_t t = blockIdx.x; t < T; t += gridDim.x) {
         // a CTA with a further row refills its shared-memory part only once every thread has read the last one
         if (RECOMPUTE && t != blockIdx.x) __syncthreads();
-        grad_row<THREADS, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef,
-                                                  eps, grad, token_loss, flags, threadIdx.x, part, part_mx, par, kp);
+        grad_row<THREADS, UNROLL, RECOMPUTE, ENT, TM>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy,
+                                                      ent_coef, eps, grad, token_loss, flags, threadIdx.x, part, part_mx,
+                                                      par, kp);
     }
-    if (RECOMPUTE && kp.tm_chunks > 0) {   // every tensor-memory read has completed (tmem_wait_ld)
-        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        __syncthreads();
-        if (warp == 0) {
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(kTmemCols)
-                         : "memory");
+    if constexpr (TM) {
+        if (kp.tm_chunks > 0) {   // every tensor-memory read has completed (tmem_wait_ld)
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncthreads();
+            if (warp == 0) {
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                             "r"(kTmemCols)
+                             : "memory");
+            }
         }
     }
 }
@@ -476,7 +508,7 @@ __global__ void __launch_bounds__(THREADS) loss_grad_warp(
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     int par = 0;
     for (int64_t t = int64_t(blockIdx.x) * NW + wid; t < T; t += int64_t(gridDim.x) * NW)
-        grad_row<32, UNROLL, RECOMPUTE, ENT>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps,
+        grad_row<32, UNROLL, RECOMPUTE, ENT, false>(logits, t, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps,
                                              grad, token_loss, flags, lane, nullptr, nullptr, par,
                                              RowKeep{nullptr, 0, 0u, 0, nullptr});
 }
@@ -522,6 +554,24 @@ acrl_status launch_loss_grad(const acrl_bf16* logits, int64_t T, int V, int64_t 
     } else if (!RECOMPUTE && V >= kWideRowMinV) {
         loss_grad_cta<kWideThreads, kCtaUnroll, false, ENT><<<unsigned(grid_for(1, T)), kWideThreads, 0, s>>>(
             logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
+    } else if (RECOMPUTE && (V >> 3) <= kSmallMaxVecs) {
+        if constexpr (RECOMPUTE) {
+            auto kernel = loss_grad_cta<kSmallThreads, kCtaUnroll, true, ENT>;
+            const int smem = 16 * min(V >> 3, kSmallKeepVecs);
+            if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+                return ACRL_ERR_CUDA;
+            kernel<<<unsigned(grid_for(1, T)), kSmallThreads, smem, s>>>(
+                logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
+        }
+    } else if (RECOMPUTE && (V >> 3) >= kTmemMinVecs) {
+        if constexpr (RECOMPUTE) {
+            auto kernel = loss_grad_cta<kCtaThreads, kCtaUnroll, true, ENT, true>;
+            const int smem = 16 * kKeepVecs;
+            if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+                return ACRL_ERR_CUDA;
+            kernel<<<unsigned(grid_for(1, T)), kCtaThreads, smem, s>>>(
+                logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
+        }
     } else {
         auto kernel = loss_grad_cta<kCtaThreads, kCtaUnroll, RECOMPUTE, ENT>;
         const int smem = RECOMPUTE ? 16 * (V >> 3 < kKeepVecs ? V >> 3 : kKeepVecs) : 0;
