@@ -342,9 +342,9 @@ acrl_status acrl_controller_step(acrl_controller_state* state, const acrl_params
  *   ids, mask  as for acrl_token_stats.
  *   lse     device float [T] from acrl_token_stats on the same logits, or
  *           NULL to recompute it here (the cached-old path: a second sweep
- *           over each row; for rows of more than 16,384 columns each CTA
- *           keeps up to 72 KB (rows of up to 40,967 columns) or 96 KB of its
- *           row in shared memory, loaded by one bulk copy per row whose wait
+ *           over each row; for rows of more than 6,144 columns each CTA
+ *           keeps up to 40 KB (rows of up to 24,583 columns), 72 KB (up to
+ *           40,967) or 96 KB of its row in shared memory, loaded by one bulk copy per row whose wait
  *           is bounded (ACRL_FLAG_TIMEOUT), and, from 65,536 columns, up to
  *           128 KB in tensor memory between the sweeps: it then allocates 256
  *           of the SM's 512 tensor-memory columns while it runs).

@@ -58,7 +58,7 @@ static_assert(kCtaThreads == 512 && kCtaUnroll == 4, "column layout: 16 warps, 4
 // until it has given up its allocation permit: measured with ncu, 15.6 warps
 // resident per SM against 30.7 for the same work without tcgen05 code.
 constexpr int kTmemMinVecs = kKeepVecs + kChunk;
-// Rows of up to kSmallMaxVecs vectors (V <= 40,967) take 256-thread CTAs in
+// Longer rows of up to kSmallMaxVecs vectors (V <= 40,967) take 256-thread CTAs in
 // the recompute path, each keeping up to 72 KB of its row in shared memory so
 // that three fit on an SM (the rest of the row, at most 8 KB, is read again
 // from L2): 0.92-0.98 of the copy rate for V = 32,000-40,000 against 0.77-0.85
@@ -67,6 +67,21 @@ constexpr int kTmemMinVecs = kKeepVecs + kChunk;
 constexpr int kSmallThreads = 256;
 constexpr int kSmallKeepVecs = 4608;
 constexpr int kSmallMaxVecs = 5120;
+// Rows of up to kTinyMaxVecs vectors (V <= 24,583) take 128-thread CTAs that
+// keep up to 40 KB of the row (five or more CTAs per SM; the rest, at most
+// 8 KB, is read again from L2): 0.95-1.04 of the copy rate for V = 8,192-
+// 24,576, where one warp per row, reading the whole row again from L2, reached
+// 0.70-0.87 (32 rows of 32 KB in flight per SM no longer fit in L2 at
+// V = 16,384).  Rows of up to kRecomputeWarpMaxV columns keep one warp per
+// row (0.95 against 0.82 at V = 6,144).
+constexpr int kTinyThreads = 128;
+constexpr int kTinyKeepVecs = 2560;
+constexpr int kTinyMaxVecs = 3072;
+constexpr int kRecomputeWarpMaxV = 6144;
+
+// Vectors of a row that a recompute CTA of THREADS threads keeps in shared memory.
+template <int THREADS>
+constexpr int kKeepOf = THREADS == kTinyThreads ? kTinyKeepVecs : THREADS == kSmallThreads ? kSmallKeepVecs : kKeepVecs;
 
 // Where the vectors of a row live between the two sweeps of the recompute
 // path: [0, s) in `smem` (filled by a bulk copy that completes on `bar`),
@@ -451,7 +466,7 @@ __global__ void __launch_bounds__(THREADS) loss_grad_cta(
     RowKeep kp{keep, 0, 0u, 0, &keep_bar};
     if (RECOMPUTE) {
         const int nvec = V >> 3;
-        kp.s = min(THREADS == kSmallThreads ? kSmallKeepVecs : kKeepVecs, nvec);
+        kp.s = min(kKeepOf<THREADS>, nvec);
         kp.tm_chunks = TM && nvec > kKeepVecs ? min(kTmemChunks, (nvec - kKeepVecs) / kChunk) : 0;
         if (threadIdx.x == 0) {
             mbar_init(&keep_bar, 1);
@@ -547,13 +562,22 @@ acrl_status launch_loss_grad(const acrl_bf16* logits, int64_t T, int V, int64_t 
                              const uint8_t* mask, const float* lse, const float* old_logp, const float* coef,
                              const float* entropy, const float* ent_coef, float eps, acrl_bf16* grad,
                              float* token_loss, int32_t* flags, cudaStream_t s) {
-    if (V <= kWarpRowMaxV) {
+    if (V <= (RECOMPUTE ? kRecomputeWarpMaxV : kWarpRowMaxV)) {
         constexpr int THREADS = 256;
         loss_grad_warp<THREADS, 4, RECOMPUTE, ENT><<<unsigned(grid_for(THREADS / 32, T)), THREADS, 0, s>>>(
             logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
     } else if (!RECOMPUTE && V >= kWideRowMinV) {
         loss_grad_cta<kWideThreads, kCtaUnroll, false, ENT><<<unsigned(grid_for(1, T)), kWideThreads, 0, s>>>(
             logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
+    } else if (RECOMPUTE && (V >> 3) <= kTinyMaxVecs) {
+        if constexpr (RECOMPUTE) {
+            auto kernel = loss_grad_cta<kTinyThreads, kCtaUnroll, true, ENT>;
+            const int smem = 16 * min(V >> 3, kTinyKeepVecs);
+            if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+                return ACRL_ERR_CUDA;
+            kernel<<<unsigned(grid_for(1, T)), kTinyThreads, smem, s>>>(
+                logits, T, V, ld, ids, mask, lse, old_logp, coef, entropy, ent_coef, eps, grad, token_loss, flags);
+        }
     } else if (RECOMPUTE && (V >> 3) <= kSmallMaxVecs) {
         if constexpr (RECOMPUTE) {
             auto kernel = loss_grad_cta<kSmallThreads, kCtaUnroll, true, ENT>;
