@@ -20,6 +20,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -54,10 +55,10 @@ LAUNCHES_PER_STEP = 9
 # taken on (sha256 of the file and the headers beside it, first 16 hex digits).
 NCU_TRAFFIC = {
     # qwen_profile (8,192 rows x 151,936), the two timed launches averaged
-    "loss_grad.cu": {"src": "9232fa17eb3b4952", "bytes": 2.48963e9 + 2.43577e9, "units": 4978778112},
-    "token_stats.cu": {"src": "d1643f8219277aa2", "bytes": 2.49025e9 + 1.65e6, "units": 2489458688},
+    "loss_grad.cu": {"src": "4b1a35c24313491f", "bytes": 2.48963e9 + 2.43577e9, "units": 4978778112},
+    "token_stats.cu": {"src": "7ac940fa8a49ab39", "bytes": 2.49025e9 + 1.65e6, "units": 2489458688},
     # lmhead_profile (4,096 x 4,096 x 151,936: one band), flops as the unit
-    "lmhead.cu": {"src": "a8604f527150f0a7", "bytes": 2.1415e9 + 1.3065e9, "units": 2.0 * 4096 * 151936 * 4096},
+    "lmhead.cu": {"src": "55460513e79100db", "bytes": 2.1415e9 + 1.3065e9, "units": 2.0 * 4096 * 151936 * 4096},
 }
 
 
@@ -71,14 +72,22 @@ def _peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def _code_only(text):
+    """C/C++ source without its comments, blank lines and trailing blanks."""
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", "", text)
+    return "\n".join(line.rstrip() for line in text.splitlines() if line.strip())
+
+
 def _src_hash(name):
-    """Hash of a kernel source and every header beside it."""
+    """Hash of the code of a kernel source and of every header beside it
+    (comments left out: editing one does not change the kernel)."""
     csrc = os.path.join(ROOT, "paper_2607_24062_gb300", "csrc")
     headers = sorted(f for f in os.listdir(csrc) if f.endswith((".cuh", ".h")))
     d = hashlib.sha256()
     for f in (name, *headers):
-        with open(os.path.join(csrc, f), "rb") as fh:
-            d.update(fh.read())
+        with open(os.path.join(csrc, f), encoding="utf-8") as fh:
+            d.update(_code_only(fh.read()).encode())
     return d.hexdigest()[:16]
 
 

@@ -12,10 +12,11 @@
 // more FMA and a multiply.  Rows that carry no gradient (masked, zero
 // coefficient and no bonus, clipped) are written as zeros without reading
 // their logits.  With lse == NULL the row's log-sum-exp is first recomputed
-// by a sweep over the same row; the first kKeepVecs 16-byte vectors of the row
-// (96 KB) stay in the CTA's shared memory and the next up to kTmemVecs (128 KB)
-// in its tensor memory between the two sweeps, so that only the rest of the
-// row is read again, from L2.  The shared-memory part arrives by one bulk copy
+// by a sweep over the same row; the first 16-byte vectors of the row (up to
+// 40, 72 or 96 KB, by the CTA's size) stay in the CTA's shared memory and, for
+// rows of 65,536 columns or more, the next up to kTmemVecs (128 KB) in its
+// tensor memory between the two sweeps, so that only the rest of the row is
+// read again, from L2.  The shared-memory part arrives by one bulk copy
 // started when the row starts, while the threads load the rest.
 #include "acrl_device.cuh"
 #include "acrl_host.h"
@@ -27,10 +28,9 @@ namespace {
 
 constexpr uint32_t kSignPair = 0x80008000u;
 
-// Recompute path of the CTA kernel: vectors of a row kept in shared memory
-// between the sweeps (96 KB; two 512-thread CTAs per SM), a multiple of the
-// sweep's chunk (threads x unroll vectors) so that the folds are grouped as
-// in a sweep without it.
+// CTA kernel: 512 threads, four 16-byte vectors per thread and step.  Its
+// recompute path keeps kKeepVecs vectors of a row in shared memory between the
+// sweeps (96 KB, three whole sweep chunks; two 512-thread CTAs per SM).
 constexpr int kCtaThreads = 512, kCtaUnroll = 4;
 // The streaming path (lse given) takes 768-thread CTAs for rows of more than
 // 65,536 columns: 1.02-1.04 of the copy rate there against 0.99-1.02 with 512
@@ -460,7 +460,7 @@ __global__ void __launch_bounds__(THREADS) loss_grad_cta(
     __shared__ float part_mx[2 * (THREADS / 32)];
     __shared__ uint32_t tmem_base;
     __shared__ __align__(8) uint64_t keep_bar;
-    extern __shared__ uint4 keep[];  // recompute path: min(kKeepVecs, V / 8) vectors (dynamic size)
+    extern __shared__ uint4 keep[];  // recompute path: min(kKeepOf<THREADS>, V / 8) vectors (dynamic size)
     const int warp = threadIdx.x >> 5;
     static_assert(!TM || (RECOMPUTE && THREADS == kCtaThreads && UNROLL == kCtaUnroll), "tensor-memory layout");
     RowKeep kp{keep, 0, 0u, 0, &keep_bar};

@@ -34,3 +34,14 @@ def test_reference_arm_prints_one_json_line():
     assert f"{cb['cores']} processes" in cb["sample"]
     assert out["e2e"] == {"value": out["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
                           "d2h_bytes_per_step": 0}
+
+
+def test_traffic_key_ignores_comments_only():
+    """The DRAM-traffic table is keyed to a kernel's code: an edited comment
+    keeps the key, an edited statement changes it."""
+    import bench
+    a = "int f(int x) {  // one\n    return x + 1; /* two */\n}\n"
+    b = "// header\nint f(int x) {  // other words\n\n    return x + 1;\n}\n"
+    c = "int f(int x) {\n    return x + 2;\n}\n"
+    assert bench._code_only(a) == bench._code_only(b)
+    assert bench._code_only(a) != bench._code_only(c)
