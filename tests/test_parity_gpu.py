@@ -189,11 +189,12 @@ def test_uniform_logits_and_equal_policies():
 
 
 @pytest.mark.parametrize("beta", [0.0, 0.01])
-@pytest.mark.parametrize("V", [20011, 4099, 151936])
+@pytest.mark.parametrize("V", [20011, 4099, 32000, 49152, 151936])
 def test_old_logp_and_recomputed_lse(V, beta):
     """Cached-old path: weights from old log-probs, LSE recomputed in the gradient kernel, r != 1 with clipping
-    (CTA and warp row teams; rows held whole in shared memory between the two sweeps, and rows of which the
-    first 96 KB are held there and the rest read again from L2; with and without the entropy bonus)."""
+    (warp row teams, and CTAs of 128, 256 and 512 threads; rows held whole in shared memory between the two
+    sweeps, and rows of which the first 96 KB are held there, 128 KB more in tensor memory and the rest read
+    again from L2; with and without the entropy bonus)."""
     spec = W.small_variant(W.QWEN, name="offpolicy", n_prompts=2, group_size=4, len_lo=10, len_hi=80, V=V)
     b = _gen(spec, seed=31)
     p = acrl.Params(entropy_coeff=beta)
@@ -236,7 +237,7 @@ def test_old_logp_and_recomputed_lse(V, beta):
         assert_loss(float(loss), oloss, otl)
 
 
-@pytest.mark.parametrize("V", [4099, 20011, 151936])
+@pytest.mark.parametrize("V", [4099, 20011, 32000, 49152, 151936])
 def test_gradient_undefined_rows_on_gpu(V):
     """Readings c17 and c18 in the gradient call: a live row with a NaN or an
     infinite logit, or with a NaN old log-prob, gets a NaN gradient row and a
