@@ -131,3 +131,35 @@ def test_binding_rejects_buffers_on_different_devices():
         api._one_device((a, a))
     with pytest.raises(api.AcrlError, match="CUDA"):
         api._one_device((None,))
+
+
+def test_kernels_do_not_spill_and_fit_their_occupancy(L):
+    """The build's ptxas report: no kernel spills registers to local memory,
+    and the gradient kernels stay within the register counts their CTAs per
+    SM rely on (two 768-thread streaming CTAs need at most 42 registers a
+    thread, two 512-thread recompute CTAs at most 64)."""
+    import os
+    import re
+    path = os.path.join(build.BUILD, "ptxas.txt")
+    if not os.path.exists(path):
+        build.build(force=True)
+    text = open(path).read()
+    spills = re.findall(r"(\d+) bytes spill stores, (\d+) bytes spill loads", text)
+    assert spills, "no ptxas resource report"
+    assert all(int(a) == 0 and int(b) == 0 for a, b in spills), spills
+    regs = {}
+    name = None
+    for line in text.splitlines():
+        m = re.search(r"Compiling entry function '(\S+)'", line)
+        if m:
+            name = m.group(1)
+            continue
+        m = re.search(r"Used (\d+) registers", line)
+        if m and name:
+            regs[name] = int(m.group(1))
+            name = None
+    limits = {r"loss_grad_ctaILi768ELi4ELb0E": 42, r"loss_grad_ctaILi512ELi4ELb1E": 64}
+    for pattern, limit in limits.items():
+        found = {k: v for k, v in regs.items() if re.search(pattern, k)}
+        assert found, pattern
+        assert all(v <= limit for v in found.values()), found
