@@ -52,11 +52,11 @@ LAUNCHES_PER_STEP = 9
 # launch by the algorithmic bytes (or, for the GEMM, the flops) of each: the streaming
 # kernels' traffic grows in proportion to the rows, the GEMM's to the bands of 32 row
 # tiles (the weight is read once per band).  Valid only for the kernel source it was
-# taken on (sha256 of the file and the headers beside it, first 16 hex digits).
+# taken on (sha256 of the code, comments left out, of the file and the headers beside it; 16 hex digits).
 NCU_TRAFFIC = {
     # qwen_profile (8,192 rows x 151,936), the two timed launches averaged
-    "loss_grad.cu": {"src": "4b1a35c24313491f", "bytes": 2.48963e9 + 2.43577e9, "units": 4978778112},
-    "token_stats.cu": {"src": "7ac940fa8a49ab39", "bytes": 2.49025e9 + 1.65e6, "units": 2489458688},
+    "loss_grad.cu": {"src": "cdb6978dd51672a0", "bytes": 2.48952e9 + 2.43624e9, "units": 4978778112},
+    "token_stats.cu": {"src": "ab093ae84f126458", "bytes": 2.49026e9 + 1.62e6, "units": 2489458688},
     # lmhead_profile (4,096 x 4,096 x 151,936: one band), flops as the unit
     "lmhead.cu": {"src": "55460513e79100db", "bytes": 2.1415e9 + 1.3065e9, "units": 2.0 * 4096 * 151936 * 4096},
 }

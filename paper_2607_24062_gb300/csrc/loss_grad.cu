@@ -528,33 +528,68 @@ __global__ void __launch_bounds__(THREADS) loss_grad_warp(
                                              RowKeep{nullptr, 0, 0u, 0, nullptr});
 }
 
-// Scalar loss: sum of token losses in a fixed order.  Each thread adds float4
-// groups (four values in fp32) into two alternating fp64 accumulators, so the
-// loads pipeline and the fp64 adds are a quarter of the values; then a fixed
-// CTA tree in fp64 whose cross-warp pass runs in thread 0 alone.
-constexpr int kSumThreads = 1024;
-__global__ void __launch_bounds__(kSumThreads) loss_sum_kernel(const float* __restrict__ tl, int64_t T,
-                                                               float* __restrict__ loss) {
+// Scalar loss: sum of token losses in a fixed order, by one cluster of
+// kSumCtas CTAs (no scratch memory: the partial sums meet in distributed
+// shared memory).  CTA c sums its contiguous block of the token losses: each
+// thread adds float4 groups (four values in fp32) into two alternating fp64
+// accumulators, so the loads pipeline and the fp64 adds are a quarter of the
+// values; then a fixed CTA tree in fp64 whose cross-warp pass runs in thread 0
+// alone; CTA 0 adds the CTAs' sums in rank order.  Eight CTAs keep eight SMs'
+// loads in flight where one CTA left the reduction latency-bound (T = 524,288:
+// ~75 us on one CTA).
+constexpr int kSumThreads = 1024, kSumCtas = 8;
+
+__device__ __forceinline__ void sum_cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ double ld_peer_f64(const double* p, uint32_t rank) {
+    uint32_t a;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(p)), "r"(rank));
+    double v;
+    asm volatile("ld.shared::cluster.f64 %0, [%1];" : "=d"(v) : "r"(a) : "memory");
+    return v;
+}
+
+__global__ void __cluster_dims__(kSumCtas, 1, 1) __launch_bounds__(kSumThreads)
+    loss_sum_kernel(const float* __restrict__ tl, int64_t T, float* __restrict__ loss) {
     __shared__ double sh[kSumThreads / 32 * 2];
+    __shared__ double cta_sum;
+    const int64_t c = blockIdx.x;   // the launch is one cluster: the block index is the rank
     double s0 = 0.0, s1 = 0.0;
-    const bool vec = (reinterpret_cast<uintptr_t>(tl) & 15u) == 0;
-    const int64_t n4 = vec ? T / 4 : 0;
-    const float4* v = reinterpret_cast<const float4*>(tl);
-    int64_t i = threadIdx.x;
+    if ((reinterpret_cast<uintptr_t>(tl) & 15u) == 0) {
+        const int64_t n4 = T / 4;
+        const int64_t per = (n4 + kSumCtas - 1) / kSumCtas;
+        const int64_t lo = min(n4, c * per), hi = min(n4, lo + per);
+        const float4* v = reinterpret_cast<const float4*>(tl);
+        int64_t i = lo + threadIdx.x;
 #pragma unroll 4
-    for (; i + kSumThreads < n4; i += 2 * kSumThreads) {
-        const float4 a = v[i], b = v[i + kSumThreads];
-        s0 += double((a.x + a.y) + (a.z + a.w));
-        s1 += double((b.x + b.y) + (b.z + b.w));
+        for (; i + kSumThreads < hi; i += 2 * kSumThreads) {
+            const float4 a = v[i], b = v[i + kSumThreads];
+            s0 += double((a.x + a.y) + (a.z + a.w));
+            s1 += double((b.x + b.y) + (b.z + b.w));
+        }
+        for (; i < hi; i += kSumThreads) {
+            const float4 a = v[i];
+            s0 += double((a.x + a.y) + (a.z + a.w));
+        }
+        if (c == kSumCtas - 1)
+            for (int64_t j = 4 * n4 + threadIdx.x; j < T; j += kSumThreads) s1 += tl[j];
+    } else {
+        const int64_t per = (T + kSumCtas - 1) / kSumCtas;
+        const int64_t lo = min(T, c * per), hi = min(T, lo + per);
+        for (int64_t j = lo + threadIdx.x; j < hi; j += kSumThreads) s0 += tl[j];
     }
-    for (; i < n4; i += kSumThreads) {
-        const float4 a = v[i];
-        s0 += double((a.x + a.y) + (a.z + a.w));
-    }
-    for (int64_t j = 4 * n4 + threadIdx.x; j < T; j += kSumThreads) s1 += tl[j];
     double total[1] = {s0 + s1}, unused = 0.0;
     block_sums_max0<kSumThreads / 32, 1>(total, unused, sh);
-    if (threadIdx.x == 0) *loss = float(total[0]);
+    if (threadIdx.x == 0) cta_sum = total[0];
+    sum_cluster_sync();   // every CTA's sum is in its shared memory
+    if (c == 0 && threadIdx.x == 0) {
+        double r = 0.0;
+        for (uint32_t k = 0; k < uint32_t(kSumCtas); ++k) r += ld_peer_f64(&cta_sum, k);
+        *loss = float(r);
+    }
+    sum_cluster_sync();   // no CTA leaves while CTA 0 may still read its shared memory
 }
 
 template <bool RECOMPUTE, bool ENT>
@@ -642,12 +677,12 @@ extern "C" acrl_status acrl_loss_grad_logits(const acrl_bf16* logits, int64_t T,
                                               clip_eps, grad, token_loss, dev_flags, s);
         if (st != ACRL_OK) return st;
     }
-    loss_sum_kernel<<<1, kSumThreads, 0, s>>>(token_loss, T, loss);
+    loss_sum_kernel<<<kSumCtas, kSumThreads, 0, s>>>(token_loss, T, loss);
     return launch_status();
 }
 
 extern "C" acrl_status acrl_reduce_loss(const float* token_loss, int64_t T, float* loss, acrl_stream stream) {
     if (T < 0 || !loss || (T > 0 && !token_loss)) return ACRL_ERR_INVALID_ARG;
-    loss_sum_kernel<<<1, kSumThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(token_loss, T, loss);
+    loss_sum_kernel<<<kSumCtas, kSumThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(token_loss, T, loss);
     return launch_status();
 }

@@ -738,12 +738,13 @@ def test_importance_weights_from_log_probs(mode):
         assert_close_rel(api.read_state(state)["X"], ostate.X, floor=1e-12, what="X")
 
 
-@pytest.mark.parametrize("V", [1, 7, 8, 9, 6144, 6151, 6152, 16383, 16384, 16385, 20480, 24576, 24583, 24584,
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 4096, 4097, 6144, 6151, 6152, 16383, 16384, 16385, 20480, 24576, 24583, 24584,
                                32000, 36864, 36871, 36872, 40960, 40967, 40968, 49152, 49153, 49160, 65535, 65536,
                                65537, 65544, 81920, 100000, 114688, 114695])
 def test_row_size_class_boundaries(V):
-    """Vocabularies at the edges of the row-team size classes (one warp up to
-    16,384 columns, 64 threads up to 65,536, 128 above for the statistics;
+    """Vocabularies at the edges of the row-team size classes (eight lanes up
+    to 4,096 columns, one warp up to 16,384, 64 threads up to 65,536, 128
+    above for the statistics;
     one warp, then 512 threads, then 768 above 65,536 for the gradient; one
     warp up to 6,144 columns, 128 threads up to 24,583, 256 up to 40,967,
     then 512 for the gradient with the lse recomputed), of the 8-column
