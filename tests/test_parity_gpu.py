@@ -780,3 +780,24 @@ def test_row_size_class_boundaries(V):
         assert_grad_rows(grad_rows(grad, np.arange(T), V), want, host(coef), host(ids), what=f"grad (recompute "
                          f"{recompute})")
     assert api.read_flags(flags) == 0
+
+
+@pytest.mark.parametrize("offset", [0, 1])
+def test_loss_sum_blocks_tails_and_alignment(offset):
+    """acrl_reduce_loss (the scalar loss of Eq. ACRL's sum over tokens):
+    lengths at the edges of the eight CTAs' blocks of float4 groups and of the
+    ragged tail, from a 16-byte-aligned array and from one starting an element
+    later (the scalar path): the fp32 result agrees with math.fsum of the same
+    values within the rounding of fp32 groups of four, and two calls agree
+    bit for bit."""
+    gen = torch.Generator(device=DEV).manual_seed(5 + offset)
+    base = torch.randn(600_000, generator=gen, device=DEV)
+    for T in (0, 1, 3, 4, 5, 31, 32, 33, 1023, 1024, 1025, 32767, 32768, 32769, 147831, 524288 + 7):
+        x = base[offset: offset + T]
+        a = api.reduce_loss(x)
+        b = api.reduce_loss(x)
+        torch.cuda.synchronize()
+        assert torch.equal(a, b), T
+        ref = math.fsum(host(x).astype(np.float64).tolist())
+        bound = 1e-6 * float(host(x).astype(np.float64).__abs__().sum()) + 1e-6
+        assert abs(float(a) - ref) <= bound, (T, float(a), ref)
