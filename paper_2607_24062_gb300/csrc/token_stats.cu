@@ -3,10 +3,10 @@
 //
 // Each row is read exactly once from HBM with 16-byte non-allocating loads.
 // A team of threads (eight lanes for rows of up to 4,096 columns, a warp for
-// other short rows, the whole CTA for vocabulary-size rows) owns a row; every thread keeps an online base-2 state
-// (max, sum 2^(u-U), sum 2^(u-U)(u-U)) over its strided share of the row, and
-// the team merges the states with a fixed butterfly/tree order, so results
-// are bit-reproducible run to run.
+// other short rows, the whole CTA for vocabulary-size rows) owns a row; every
+// thread keeps an online base-2 state (max, sum 2^(u-U), sum 2^(u-U)(u-U))
+// over its strided share of the row, and the team merges the states with a
+// fixed butterfly/tree order, so results are bit-reproducible run to run.
 #include "acrl_device.cuh"
 #include "acrl_host.h"
 #include "row_lse.cuh"
